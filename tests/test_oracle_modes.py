@@ -1,0 +1,127 @@
+"""Pins of the oracle's computation modes: full (Algorithm 1), surrogate (§4.3), mean."""
+import math
+
+import numpy as np
+import scipy.special
+import scipy.stats
+import torch
+
+import oracle
+
+
+def test_full_attention_matches_library_sdpa():
+    g = np.random.default_rng(0)
+    for N, d in ((1, 64), (5, 4), (300, 64), (257, 16)):
+        Q, K, V = (g.standard_normal((N, d)) * 2 for _ in range(3))
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            *(torch.from_numpy(a)[None, None] for a in (Q, K, V)))[0, 0].numpy()
+        np.testing.assert_allclose(oracle.full_attention(Q, K, V), ref, rtol=1e-11, atol=1e-12)
+
+
+def test_full_attention_brute_force_tiny():
+    # Element-by-element definition on a 3-token, 2-channel problem.
+    Q = np.array([[1.0, 0.0], [0.0, 2.0], [1.0, -1.0]])
+    K = np.array([[0.5, 1.0], [-1.0, 0.0], [2.0, 1.0]])
+    V = np.array([[1.0, 2.0], [3.0, -1.0], [0.0, 4.0]])
+    out = oracle.full_attention(Q, K, V)
+    for i in range(3):
+        logits = [sum(Q[i, c] * K[j, c] for c in range(2)) / math.sqrt(2) for j in range(3)]
+        w = [math.exp(x) for x in logits]
+        z = sum(w)
+        for c in range(2):
+            assert abs(out[i, c] - sum(w[j] / z * V[j, c] for j in range(3))) < 1e-14
+
+
+def test_full_attention_special_cases():
+    g = np.random.default_rng(1)
+    N, d = 200, 64
+    Q, V = g.standard_normal((N, d)), g.standard_normal((N, d))
+    # Identical keys: uniform weights, every row is the mean of V.
+    K = np.tile(g.standard_normal(d), (N, 1))
+    np.testing.assert_allclose(oracle.full_attention(Q, K, V), np.tile(V.mean(0), (N, 1)), rtol=1e-12, atol=1e-13)
+    # Constant V: output equals V.
+    Vc = np.tile(g.standard_normal(d), (N, 1))
+    np.testing.assert_allclose(oracle.full_attention(Q, g.standard_normal((N, d)), Vc), Vc, rtol=1e-12)
+    # V = identity (d = N): the output is the attention matrix; rows sum to one.
+    n = 40
+    P = oracle.full_attention(g.standard_normal((n, n)), g.standard_normal((n, n)), np.eye(n))
+    np.testing.assert_allclose(P.sum(1), 1.0, atol=1e-13)
+    assert np.all(P > 0)
+    # Row subset equals the same rows of the full computation.
+    Kr = g.standard_normal((N, d))
+    rows = np.array([0, 17, 199, 5])
+    np.testing.assert_allclose(oracle.full_attention(Q, Kr, V, rows=rows), oracle.full_attention(Q, Kr, V)[rows], rtol=1e-13)
+
+
+def _mlp_params(g, d, L, zero_out=False):
+    W1, b1 = g.standard_normal((L, 2 * d)) * 0.3, g.standard_normal(L) * 0.1
+    W2, b2 = g.standard_normal((d, L)) * 0.3, g.standard_normal(d) * 0.1
+    if zero_out:
+        W2, b2 = np.zeros_like(W2), np.zeros_like(b2)
+    return W1, b1, W2, b2
+
+
+def test_surrogate_without_correction_is_single_query_attention():
+    g = np.random.default_rng(2)
+    N, d, L = 500, 64, 64
+    V = g.standard_normal((N, d))
+    r = oracle.softmax(g.standard_normal(N) * 4)
+    y, C = oracle.surrogate_attention(V, r, _mlp_params(g, d, L), _mlp_params(g, d, L, zero_out=True))
+    # delta = 0 -> y = C_h = r_h V_h for every token.
+    np.testing.assert_allclose(C, (V * r[:, None]).sum(0), rtol=1e-12)
+    np.testing.assert_allclose(y, np.tile(C, (N, 1)), rtol=1e-12)
+    # One-hot routing vector: C_h is that token's value.
+    onehot = np.zeros(N)
+    onehot[123] = 1.0
+    _, C1 = oracle.surrogate_attention(V, onehot, _mlp_params(g, d, L), _mlp_params(g, d, L, zero_out=True))
+    np.testing.assert_array_equal(C1, V[123])
+
+
+def test_surrogate_concatenation_order_gate_and_activation():
+    # z = [v_i, C_h].  MLP_delta's first layer picks the v half (W1 = [I | 0]), its
+    # second layer is the identity; MLP_gamma has a zero output layer, so
+    # gamma = sigma(0) = 1/2.  Then y_i = C_h + 1/2 * v_i * Phi(v_i) channel-wise.
+    g = np.random.default_rng(3)
+    N, d = 64, 8
+    V = g.standard_normal((N, d)) * 2
+    r = oracle.softmax(g.standard_normal(N))
+    C = (V * r[:, None]).sum(0)
+    I = np.eye(d)
+    pick_v = (np.concatenate([I, np.zeros((d, d))], 1), np.zeros(d), I, np.zeros(d))
+    pick_c = (np.concatenate([np.zeros((d, d)), I], 1), np.zeros(d), I, np.zeros(d))
+    gamma0 = (np.zeros((d, 2 * d)), np.zeros(d), np.zeros((d, d)), np.zeros(d))
+    y, _ = oracle.surrogate_attention(V, r, gamma0, pick_v)
+    np.testing.assert_allclose(y, C + 0.5 * V * scipy.stats.norm.cdf(V), rtol=1e-12, atol=1e-13)
+    # Picking the context half makes the correction identical for every token.
+    y2, _ = oracle.surrogate_attention(V, r, gamma0, pick_c)
+    np.testing.assert_allclose(y2, np.tile(C + 0.5 * C * scipy.stats.norm.cdf(C), (N, 1)), rtol=1e-12)
+    # A gate MLP whose output bias is b gives gamma = expit(b) channel-wise.
+    b = np.linspace(-3, 3, d)
+    gamma_b = (np.zeros((d, 2 * d)), np.zeros(d), np.zeros((d, d)), b)
+    y3, _ = oracle.surrogate_attention(V, r, gamma_b, pick_v)
+    np.testing.assert_allclose(y3, C + scipy.special.expit(b) * V * scipy.stats.norm.cdf(V), rtol=1e-12, atol=1e-13)
+
+
+def test_surrogate_rows_subset():
+    g = np.random.default_rng(4)
+    V = g.standard_normal((100, 64))
+    r = oracle.softmax(g.standard_normal(100))
+    mg, md = _mlp_params(g, 64, 64), _mlp_params(g, 64, 64)
+    full, _ = oracle.surrogate_attention(V, r, mg, md)
+    rows = [3, 99, 0]
+    sub, _ = oracle.surrogate_attention(V, r, mg, md, rows=rows)
+    np.testing.assert_allclose(sub, full[rows], rtol=1e-12, atol=1e-14)
+
+
+def test_mean_pooling_closed_forms():
+    g = np.random.default_rng(5)
+    v = g.standard_normal(64)
+    Vc = np.tile(v, (333, 1))
+    y, mu = oracle.mean_pooling(Vc)
+    np.testing.assert_allclose(y, Vc, rtol=1e-14)
+    A, B = g.standard_normal((50, 64)), g.standard_normal((50, 64))
+    ya, _ = oracle.mean_pooling(A)
+    yb, _ = oracle.mean_pooling(B)
+    yab, _ = oracle.mean_pooling(2 * A - 3 * B)
+    np.testing.assert_allclose(yab, 2 * ya - 3 * yb, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(ya[0], A.mean(0), rtol=1e-13)
