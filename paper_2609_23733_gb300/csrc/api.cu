@@ -1,0 +1,459 @@
+// C ABI of the library (include/vp.h): argument checks, workspace carving, launches.
+// Every entry point validates its arguments on the host before it enqueues anything and
+// returns a vp_status; kernels run on the caller's stream and nothing here synchronises
+// the host (except vp_read_device_error, whose purpose is to read the device error word).
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "internal.h"
+#include "vp.h"
+
+namespace vp {
+
+// ------------------------------------------------------------------ device queries
+namespace {
+struct DevInfo {
+  int sms = 0;
+  int sm103 = -1;
+};
+DevInfo g_dev[64];
+std::mutex g_dev_mu;
+
+DevInfo& dev_info() {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  DevInfo& d = g_dev[dev & 63];
+  if (d.sm103 < 0) {
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
+    d.sm103 = (major == 10 && minor == 3) ? 1 : 0;
+  }
+  return d;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn g_encode = nullptr;
+std::once_flag g_encode_once;
+}  // namespace
+
+int device_sm_count() { return dev_info().sms; }
+bool device_is_sm103() { return dev_info().sm103 == 1; }
+
+cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
+                              uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows) {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+  });
+  if (!g_encode) return cudaErrorNotSupported;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {pitch_elems * 2};
+  const cuuint32_t box[2] = {box_cols, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace vp
+
+using namespace vp;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+vp_status check_dims(const vp_dims* dm) {
+  if (!dm) return VP_ERR_INVALID_ARG;
+  if (dm->d != kHeadDim || dm->L != kHidden || dm->H < 1 || dm->H > kMaxHeads || dm->N < 1)
+    return VP_ERR_UNSUPPORTED_SHAPE;
+  if (!(dm->tau_low == dm->tau_low) || !(dm->tau_high == dm->tau_high)) return VP_ERR_INVALID_ARG;
+  return VP_OK;
+}
+
+vp_status check_device() {
+  if (!device_is_sm103()) return VP_ERR_UNSUPPORTED_DEVICE;
+  return VP_OK;
+}
+
+size_t layer_ws_bytes(const vp_dims* dm) {
+  const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
+  return router_scratch_bytes(dm->H) + align_up(N * 3 * D * 2) + align_up(N * D * 2);
+}
+
+size_t stack_ws_bytes(const vp_dims* dm) {
+  const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
+  // x~ (LN output) + one region shared by {QKV, Y} and the FFN hidden layer.
+  return router_scratch_bytes(dm->H) + align_up(N * D * 2) + align_up(N * 4 * D * 2);
+}
+
+// Row widths the LayerNorm kernel is instantiated for.
+bool ln_width_supported(int D) {
+  return D == 256 || D == 512 || D == 768 || D == 1024 || D == 2048 || D == 4096;
+}
+
+vp_status from_cuda(cudaError_t e) { return e == cudaSuccess ? VP_OK : VP_ERR_CUDA; }
+
+#define VP_TRY(x)                      \
+  do {                                 \
+    vp_status _s = (x);                \
+    if (_s != VP_OK) return _s;        \
+  } while (0)
+
+vp_status check_router_weights(const vp_router_weights* rw) {
+  if (!rw || !rw->W || !rw->U || !rw->w) return VP_ERR_INVALID_ARG;
+  if (!aligned16(rw->W) || !aligned16(rw->U)) return VP_ERR_ALIGNMENT;
+  return VP_OK;
+}
+
+vp_status check_surrogate_weights(const vp_surrogate_weights* sw) {
+  if (!sw || !sw->g1_w || !sw->g1_b || !sw->g2_w || !sw->g2_b || !sw->d1_w || !sw->d1_b ||
+      !sw->d2_w || !sw->d2_b)
+    return VP_ERR_INVALID_ARG;
+  if (!aligned16(sw->g1_w) || !aligned16(sw->g2_w) || !aligned16(sw->d1_w) || !aligned16(sw->d2_w))
+    return VP_ERR_ALIGNMENT;
+  return VP_OK;
+}
+
+RouterArgs make_router_args(const vp_dims* dm, const vp_bf16* qkv, const vp_router_weights* rw,
+                            const int32_t* force_modes) {
+  RouterArgs a{};
+  a.N = dm->N;
+  a.H = dm->H;
+  a.tau_low = dm->tau_low;
+  a.tau_high = dm->tau_high;
+  a.qkv = reinterpret_cast<const __nv_bfloat16*>(qkv);
+  a.W = reinterpret_cast<const __nv_bfloat16*>(rw->W);
+  a.U = reinterpret_cast<const __nv_bfloat16*>(rw->U);
+  a.w = reinterpret_cast<const __nv_bfloat16*>(rw->w);
+  a.bW = rw->bW;
+  a.bU = rw->bU;
+  a.beta = rw->beta;
+  a.force_modes = force_modes;
+  return a;
+}
+
+SurrogateArgs make_surrogate_args(const vp_surrogate_weights* sw) {
+  SurrogateArgs s;
+  s.g1_w = reinterpret_cast<const __nv_bfloat16*>(sw->g1_w);
+  s.g1_b = sw->g1_b;
+  s.g2_w = reinterpret_cast<const __nv_bfloat16*>(sw->g2_w);
+  s.g2_b = sw->g2_b;
+  s.d1_w = reinterpret_cast<const __nv_bfloat16*>(sw->d1_w);
+  s.d1_b = sw->d1_b;
+  s.d2_w = reinterpret_cast<const __nv_bfloat16*>(sw->d2_w);
+  s.d2_b = sw->d2_b;
+  return s;
+}
+
+// Runs the three mode kernels for bins already in device memory.
+vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* head_ids,
+                    const int32_t* offsets, const float* ctx, const float* mean_v,
+                    const vp_surrogate_weights* sw, __nv_bfloat16* y, unsigned int* err,
+                    cudaStream_t st) {
+  HeadAttnArgs ha{};
+  ha.N = dm->N;
+  ha.H = dm->H;
+  ha.qkv = qkv;
+  ha.head_ids = head_ids;
+  ha.offsets = offsets;
+  ha.ctx = ctx;
+  ha.mean_v = mean_v;
+  ha.sw = make_surrogate_args(sw);
+  ha.y = y;
+  ha.err = err;
+  const int sms = device_sm_count();
+  VP_TRY(from_cuda(launch_full_heads(ha, sms, st)));
+  VP_TRY(from_cuda(launch_surrogate_heads(ha, sms, st)));
+  VP_TRY(from_cuda(launch_mean_heads(ha, sms, st)));
+  return VP_OK;
+}
+
+// QKV projection -> router -> bins -> heads -> W_O (+ optional LayerScale / residual).
+vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* w_qkv,
+                    const float* b_qkv, const vp_bf16* w_o, const float* b_o, const float* ls1,
+                    const __nv_bfloat16* residual, const vp_router_weights* rw,
+                    const vp_surrogate_weights* sw, const int32_t* force_modes,
+                    __nv_bfloat16* out, __nv_bfloat16* qkv, __nv_bfloat16* y, float* s_out,
+                    int32_t* modes_out, const RouterScratch& sc, cudaStream_t st) {
+  const int N = dm->N, D = dm->H * kHeadDim;
+  const int sms = device_sm_count();
+  LinearArgs la{};
+  la.M = N;
+  la.N = 3 * D;
+  la.K = D;
+  la.A = xin;
+  la.W = reinterpret_cast<const __nv_bfloat16*>(w_qkv);
+  la.bias = b_qkv;
+  la.act = VP_ACT_NONE;
+  la.out = qkv;
+  la.err = sc.err;
+  VP_TRY(from_cuda(launch_linear(la, sms, st)));
+  RouterArgs ra = make_router_args(dm, reinterpret_cast<const vp_bf16*>(qkv), rw, force_modes);
+  ra.s_out = s_out;
+  ra.modes_out = modes_out;
+  VP_TRY(from_cuda(launch_router(ra, sc, sms, st)));
+  VP_TRY(run_heads(dm, qkv, sc.head_ids, sc.offsets, sc.ctx, sc.mean_v, sw, y, sc.err, st));
+  LinearArgs lo{};
+  lo.M = N;
+  lo.N = D;
+  lo.K = D;
+  lo.A = y;
+  lo.W = reinterpret_cast<const __nv_bfloat16*>(w_o);
+  lo.bias = b_o;
+  lo.act = VP_ACT_NONE;
+  lo.scale = ls1;
+  lo.residual = residual;
+  lo.out = out;
+  lo.err = sc.err;
+  VP_TRY(from_cuda(launch_linear(lo, sms, st)));
+  return VP_OK;
+}
+
+__device__ unsigned int g_linear_err;  // error word of vp_linear (it has no workspace)
+
+}  // namespace
+
+extern "C" {
+
+const char* vp_status_string(vp_status s) {
+  switch (s) {
+    case VP_OK: return "ok";
+    case VP_ERR_INVALID_ARG: return "invalid argument";
+    case VP_ERR_UNSUPPORTED_SHAPE: return "unsupported shape";
+    case VP_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
+    case VP_ERR_CUDA: return "CUDA error";
+    case VP_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+    case VP_ERR_WORKSPACE: return "workspace missing or too small";
+    case VP_ERR_UNSUPPORTED_DEVICE: return "device is not sm_103";
+  }
+  return "unknown status";
+}
+
+vp_status vp_workspace_size(const vp_dims* dims, int32_t what, size_t* bytes) {
+  VP_TRY(check_dims(dims));
+  if (!bytes) return VP_ERR_INVALID_ARG;
+  switch (what) {
+    case VP_WS_ROUTER: *bytes = router_scratch_bytes(dims->H); break;
+    case VP_WS_LAYER: *bytes = layer_ws_bytes(dims); break;
+    case VP_WS_STACK: *bytes = stack_ws_bytes(dims); break;
+    default: return VP_ERR_INVALID_ARG;
+  }
+  return VP_OK;
+}
+
+vp_status vp_read_device_error(void* ws, size_t ws_bytes, uint32_t* host_bits, void* stream) {
+  if (!ws || !host_bits || ws_bytes < 256) return VP_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t bits = 0;
+  if (cudaMemcpyAsync(&bits, ws, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess) return VP_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return VP_ERR_CUDA;
+  if (cudaMemsetAsync(ws, 0, 4, st) != cudaSuccess) return VP_ERR_CUDA;
+  *host_bits = bits;
+  return (bits & VP_DEVERR_WAIT_TIMEOUT) ? VP_ERR_DEVICE_TIMEOUT : VP_OK;
+}
+
+vp_status vp_router(const vp_dims* dims, const vp_bf16* qkv, const vp_router_weights* rw,
+                    const int32_t* force_modes, float* s, int32_t* modes, float* q_pool,
+                    float* ctx, float* mean_v, float* r, void* ws, size_t ws_bytes, void* stream) {
+  VP_TRY(check_dims(dims));
+  if (!qkv || !s || !modes) return VP_ERR_INVALID_ARG;
+  if (!aligned16(qkv)) return VP_ERR_ALIGNMENT;
+  VP_TRY(check_router_weights(rw));
+  if (!ws || ws_bytes < router_scratch_bytes(dims->H)) return VP_ERR_WORKSPACE;
+  VP_TRY(check_device());
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  RouterScratch sc = carve_router_scratch(ws, dims->H);
+  RouterArgs a = make_router_args(dims, qkv, rw, force_modes);
+  a.s_out = s;
+  a.modes_out = modes;
+  a.q_pool_out = q_pool;
+  a.ctx_out = ctx;
+  a.mean_v_out = mean_v;
+  a.r_out = r;
+  return from_cuda(launch_router(a, sc, device_sm_count(), st));
+}
+
+vp_status vp_bin_heads(int32_t H, int32_t N, const int32_t* modes, int32_t* head_ids,
+                       int32_t* offsets, int32_t* work, int32_t* n_work, void* stream) {
+  if (H < 1 || H > kMaxHeads || N < 1) return VP_ERR_UNSUPPORTED_SHAPE;
+  if (!modes || !head_ids || !offsets) return VP_ERR_INVALID_ARG;
+  VP_TRY(check_device());
+  return from_cuda(launch_bin_heads(H, N, modes, head_ids, offsets, work, n_work,
+                                    static_cast<cudaStream_t>(stream)));
+}
+
+vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32_t* head_ids,
+                            const int32_t* offsets, const float* ctx, const float* mean_v,
+                            const vp_surrogate_weights* sw, vp_bf16* y, void* ws, size_t ws_bytes,
+                            void* stream) {
+  VP_TRY(check_dims(dims));
+  if (!qkv || !head_ids || !offsets || !ctx || !mean_v || !y) return VP_ERR_INVALID_ARG;
+  if (!aligned16(qkv) || !aligned16(y)) return VP_ERR_ALIGNMENT;
+  VP_TRY(check_surrogate_weights(sw));
+  if (!ws || ws_bytes < router_scratch_bytes(dims->H)) return VP_ERR_WORKSPACE;
+  VP_TRY(check_device());
+  RouterScratch sc = carve_router_scratch(ws, dims->H);
+  return run_heads(dims, reinterpret_cast<const __nv_bfloat16*>(qkv), head_ids, offsets, ctx,
+                   mean_v, sw, reinterpret_cast<__nv_bfloat16*>(y), sc.err,
+                   static_cast<cudaStream_t>(stream));
+}
+
+vp_status vp_linear(int32_t M, int32_t Nout, int32_t K, const vp_bf16* A, const vp_bf16* W,
+                    const float* bias, int32_t act, const float* scale, const vp_bf16* residual,
+                    vp_bf16* out, void* stream) {
+  if (M < 1 || Nout < 8 || K < 8 || Nout % 8 || K % 8) return VP_ERR_UNSUPPORTED_SHAPE;
+  if (!A || !W || !out) return VP_ERR_INVALID_ARG;
+  if (act != VP_ACT_NONE && act != VP_ACT_GELU) return VP_ERR_INVALID_ARG;
+  if (!aligned16(A) || !aligned16(W) || !aligned16(out) || (residual && !aligned16(residual)))
+    return VP_ERR_ALIGNMENT;
+  VP_TRY(check_device());
+  unsigned int* err = nullptr;
+  if (cudaGetSymbolAddress(reinterpret_cast<void**>(&err), g_linear_err) != cudaSuccess)
+    return VP_ERR_CUDA;
+  LinearArgs la{};
+  la.M = M;
+  la.N = Nout;
+  la.K = K;
+  la.A = reinterpret_cast<const __nv_bfloat16*>(A);
+  la.W = reinterpret_cast<const __nv_bfloat16*>(W);
+  la.bias = bias;
+  la.act = act;
+  la.scale = scale;
+  la.residual = reinterpret_cast<const __nv_bfloat16*>(residual);
+  la.out = reinterpret_cast<__nv_bfloat16*>(out);
+  la.err = err;
+  return from_cuda(launch_linear(la, device_sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+vp_status vp_layer_norm(int32_t M, int32_t D, const vp_bf16* x, const float* gamma,
+                        const float* beta, float eps, vp_bf16* out, void* stream) {
+  if (M < 1 || !ln_width_supported(D)) return VP_ERR_UNSUPPORTED_SHAPE;
+  if (!x || !gamma || !beta || !out) return VP_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(out)) return VP_ERR_ALIGNMENT;
+  VP_TRY(check_device());
+  return from_cuda(launch_layer_norm(M, D, reinterpret_cast<const __nv_bfloat16*>(x), gamma, beta,
+                                     eps, reinterpret_cast<__nv_bfloat16*>(out),
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const vp_bf16* w_qkv,
+                                  const float* b_qkv, const vp_bf16* w_o, const float* b_o,
+                                  const vp_router_weights* rw, const vp_surrogate_weights* sw,
+                                  const int32_t* force_modes, vp_bf16* out, vp_bf16* qkv_out,
+                                  vp_bf16* y_out, float* s_out, int32_t* modes_out, void* ws,
+                                  size_t ws_bytes, void* stream) {
+  VP_TRY(check_dims(dims));
+  if (!x || !w_qkv || !w_o || !out) return VP_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(w_o) || !aligned16(out) ||
+      (qkv_out && !aligned16(qkv_out)) || (y_out && !aligned16(y_out)))
+    return VP_ERR_ALIGNMENT;
+  VP_TRY(check_router_weights(rw));
+  VP_TRY(check_surrogate_weights(sw));
+  if (!ws || ws_bytes < layer_ws_bytes(dims)) return VP_ERR_WORKSPACE;
+  VP_TRY(check_device());
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t N = dims->N, D = (size_t)dims->H * kHeadDim;
+  RouterScratch sc = carve_router_scratch(ws, dims->H);
+  char* p = static_cast<char*>(ws) + router_scratch_bytes(dims->H);
+  __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
+  p += align_up(N * 3 * D * 2);
+  __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p);
+  if (qkv_out) qkv = reinterpret_cast<__nv_bfloat16*>(qkv_out);
+  if (y_out) y = reinterpret_cast<__nv_bfloat16*>(y_out);
+  return run_layer(dims, reinterpret_cast<const __nv_bfloat16*>(x), w_qkv, b_qkv, w_o, b_o,
+                   nullptr, nullptr, rw, sw, force_modes, reinterpret_cast<__nv_bfloat16*>(out),
+                   qkv, y, s_out, modes_out, sc, st);
+}
+
+vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
+                          const vp_layer_weights* layers, const int32_t* force_modes,
+                          int32_t* modes_out, float* s_out, float ln_eps, void* ws,
+                          size_t ws_bytes, void* stream) {
+  VP_TRY(check_dims(dims));
+  if (n_layers < 1 || !x_inout || !layers) return VP_ERR_INVALID_ARG;
+  if (!aligned16(x_inout)) return VP_ERR_ALIGNMENT;
+  const int D = dims->H * kHeadDim;
+  if (!ln_width_supported(D)) return VP_ERR_UNSUPPORTED_SHAPE;
+  for (int l = 0; l < n_layers; ++l) {
+    const vp_layer_weights& w = layers[l];
+    if (!w.ln1_g || !w.ln1_b || !w.w_qkv || !w.w_o || !w.ls1 || !w.ln2_g || !w.ln2_b ||
+        !w.w_fc1 || !w.w_fc2 || !w.ls2)
+      return VP_ERR_INVALID_ARG;
+    if (!aligned16(w.w_qkv) || !aligned16(w.w_o) || !aligned16(w.w_fc1) || !aligned16(w.w_fc2))
+      return VP_ERR_ALIGNMENT;
+    VP_TRY(check_router_weights(&w.router));
+    VP_TRY(check_surrogate_weights(&w.surrogate));
+  }
+  if (!ws || ws_bytes < stack_ws_bytes(dims)) return VP_ERR_WORKSPACE;
+  VP_TRY(check_device());
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t N = dims->N;
+  RouterScratch sc = carve_router_scratch(ws, dims->H);
+  char* p = static_cast<char*>(ws) + router_scratch_bytes(dims->H);
+  __nv_bfloat16* xt = reinterpret_cast<__nv_bfloat16*>(p);
+  p += align_up(N * D * 2);
+  __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
+  __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p + align_up(N * 3 * D * 2));
+  __nv_bfloat16* hid = reinterpret_cast<__nv_bfloat16*>(p);  // reuses the QKV / Y region
+  __nv_bfloat16* x = reinterpret_cast<__nv_bfloat16*>(x_inout);
+  const int sms = device_sm_count();
+  for (int l = 0; l < n_layers; ++l) {
+    const vp_layer_weights& w = layers[l];
+    // (1) X~ = LN1(X)
+    VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln1_g, w.ln1_b, ln_eps, xt, st)));
+    // (2)-(3) routed attention; X <- X + LS1 (Y W_O + b_O) in place
+    VP_TRY(run_layer(dims, xt, w.w_qkv, w.b_qkv, w.w_o, w.b_o, w.ls1, x, &w.router, &w.surrogate,
+                     force_modes ? force_modes + (size_t)l * dims->H : nullptr, x, qkv, y,
+                     s_out ? s_out + (size_t)l * dims->H : nullptr,
+                     modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st));
+    // (4) Z~ = LN2(X_attn); X <- X_attn + LS2 FFN(Z~)
+    VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, xt, st)));
+    LinearArgs f1{};
+    f1.M = dims->N;
+    f1.N = 4 * D;
+    f1.K = D;
+    f1.A = xt;
+    f1.W = reinterpret_cast<const __nv_bfloat16*>(w.w_fc1);
+    f1.bias = w.b_fc1;
+    f1.act = VP_ACT_GELU;
+    f1.out = hid;
+    f1.err = sc.err;
+    VP_TRY(from_cuda(launch_linear(f1, sms, st)));
+    LinearArgs f2{};
+    f2.M = dims->N;
+    f2.N = D;
+    f2.K = 4 * D;
+    f2.A = hid;
+    f2.W = reinterpret_cast<const __nv_bfloat16*>(w.w_fc2);
+    f2.bias = w.b_fc2;
+    f2.act = VP_ACT_NONE;
+    f2.scale = w.ls2;
+    f2.residual = x;
+    f2.out = x;
+    f2.err = sc.err;
+    VP_TRY(from_cuda(launch_linear(f2, sms, st)));
+  }
+  return VP_OK;
+}
+
+}  // extern "C"

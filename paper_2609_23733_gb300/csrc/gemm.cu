@@ -1,0 +1,236 @@
+// Dense projections of Algorithm 1 (QKV, W_O, FFN) on the sm_103a tensor cores:
+//   out[M][N] = residual + scale (.) act(A[M][K] W[N][K]^T + bias)
+// Persistent CTAs (one per SM), 128 x 256 output tiles, 64-wide K blocks through a 4-stage
+// TMA ring (128-byte swizzle), tcgen05.mma (M=128, N=256, K=16, bf16 -> fp32) into one of
+// two TMEM accumulators, so the epilogue of tile i overlaps the main loop of tile i+1.
+// Warp roles: warp 0 TMA, warp 1 TMEM owner + MMA issue, warps 2-5 epilogue (one row per
+// thread: TMEM lane -> registers -> bias / GELU / LayerScale / residual -> bf16 stores).
+// Tiles are visited N-fastest so the CTAs in flight share A rows and all of W in L2.
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace vp {
+
+namespace {
+
+constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
+constexpr int kABytes = kBM * kBK * 2;  // 16 KB
+constexpr int kBBytes = kBN * kBK * 2;  // 32 KB
+constexpr uint32_t kTmemCols = 512;
+
+struct GemmSmem {
+  __nv_bfloat16 a[kStages][kBM * kBK];
+  __nv_bfloat16 b[kStages][kBN * kBK];
+  uint64_t full[kStages], empty[kStages];
+  uint64_t acc_full[2], acc_empty[2], drain;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+struct GemmParams {
+  int M, N, K;
+  const float* bias;
+  int act;
+  const float* scale;
+  const __nv_bfloat16* residual;
+  __nv_bfloat16* out;
+  unsigned int* err;
+};
+
+__device__ __forceinline__ float gelu_erf(float x) {
+  return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
+}
+
+__global__ void __launch_bounds__(192, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
+                const __grid_constant__ CUtensorMap tmap_b, GemmParams prm) {
+  extern __shared__ unsigned char smem_raw[];
+  GemmSmem& sm = *reinterpret_cast<GemmSmem*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int M = prm.M, N = prm.N, K = prm.K;
+  const int m_tiles = (M + kBM - 1) / kBM, n_tiles = (N + kBN - 1) / kBN;
+  const int tiles = m_tiles * n_tiles;
+  const int k_blocks = (K + kBK - 1) / kBK;
+  if ((int)blockIdx.x >= tiles) return;
+  const int warp = warp_id(), lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.acc_full[b], 1);
+      mbar_init(&sm.acc_empty[b], 128);
+    }
+    mbar_init(&sm.drain, 1);
+    sm.abort_flag = 0;
+    fence_mbarrier_init();
+    fence_proxy_async_smem();
+    tma_prefetch_desc(&tmap_a);
+    tma_prefetch_desc(&tmap_b);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t lc = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        const int mt = t / n_tiles, nt = t - mt * n_tiles;
+        for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
+          const int st = lc % kStages;
+          ok = mbar_wait(&sm.empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
+          if (!ok) break;
+          mbar_arrive_expect_tx(&sm.full[st], kABytes + kBBytes);
+          tma_load_2d(sm.a[st], &tmap_a, &sm.full[st], kb * kBK, mt * kBM);
+          tma_load_2d(sm.b[st], &tmap_b, &sm.full[st], kb * kBK, nt * kBN);
+        }
+      }
+      if (!ok) {
+        for (int s = 0; s < kStages; ++s) {
+          if (lc > (uint32_t)s) {
+            const uint32_t last = (lc - 1 - s) / kStages * kStages + s;
+            for (int i = 0; i < 1000000 && !mbar_try_wait(&sm.full[s], (last / kStages) & 1); ++i) {}
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kBM, kBN, 0, 0);
+      uint32_t lc = 0, i = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+        const uint32_t ab = i & 1;
+        ok = mbar_wait(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1, prm.err, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t d = tmem + ab * kBN;
+        for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
+          const int st = lc % kStages;
+          ok = mbar_wait(&sm.full[st], (lc / kStages) & 1, prm.err, abort_flag);
+          if (!ok) break;
+          tc_fence_after();
+          const uint64_t da = sdesc_sw128(smem_u32(sm.a[st]));
+          const uint64_t db = sdesc_sw128(smem_u32(sm.b[st]));
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_ss(d, da + 2 * kk, db + 2 * kk, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(&sm.empty[st]);
+        }
+        if (!ok) break;
+        tc_commit(&sm.acc_full[ab]);
+      }
+      if (!ok) {
+        tc_commit(&sm.drain);
+        for (int it = 0; it < 1000000 && !mbar_try_wait(&sm.drain, 0); ++it) {}
+      }
+    }
+  } else {
+    const int quarter = warp & 3;
+    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
+    uint32_t i = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
+      const int mt = t / n_tiles, nt = t - mt * n_tiles;
+      const uint32_t ab = i & 1;
+      bool ok = mbar_wait(&sm.acc_full[ab], (i >> 1) & 1, prm.err, abort_flag);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      tc_fence_after();
+      const int row = mt * kBM + quarter * 32 + lane;
+      const bool row_ok = row < M;
+      for (int cc = 0; cc < kBN / 32; ++cc) {
+        float v[32];
+        __syncwarp();  // TMEM loads are warp-collective; lanes may have skipped a chunk
+        tmem_ld32(t_lane + ab * kBN + cc * 32, v);
+        tmem_wait_ld();
+        if (cc == kBN / 32 - 1) {
+          tc_fence_before();
+          mbar_arrive(&sm.acc_empty[ab]);
+        }
+        const int col0 = nt * kBN + cc * 32;
+        if (!row_ok || col0 >= N) continue;
+        float res[32];
+        const bool full_chunk = col0 + 32 <= N;
+        if (prm.residual) {
+          const __nv_bfloat16* rp = prm.residual + (size_t)row * N + col0;
+          if (full_chunk) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const uint4 u = *reinterpret_cast<const uint4*>(rp + 8 * q);
+              const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                res[8 * q + 2 * e] = bf16_lo(uw[e]);
+                res[8 * q + 2 * e + 1] = bf16_hi(uw[e]);
+              }
+            }
+          } else {
+            for (int e = 0; e < 32; ++e) res[e] = col0 + e < N ? __bfloat162float(rp[e]) : 0.f;
+          }
+        }
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const int col = min(col0 + e, N - 1);
+          float x = v[e];
+          if (prm.bias) x += __ldg(prm.bias + col);
+          if (prm.act == VP_ACT_GELU) x = gelu_erf(x);
+          if (prm.scale) x *= __ldg(prm.scale + col);
+          if (prm.residual) x += res[e];
+          v[e] = x;
+        }
+        __nv_bfloat16* op = prm.out + (size_t)row * N + col0;
+        if (full_chunk) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint4 u;
+            u.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
+            u.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
+            u.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
+            u.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
+            *reinterpret_cast<uint4*>(op + 8 * q) = u;
+          }
+        } else {
+          for (int e = 0; e < 32 && col0 + e < N; ++e) op[e] = __float2bfloat16_rn(v[e]);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
+  CUtensorMap ta, tb;
+  cudaError_t e = make_tmap_bf16_2d(&ta, a.A, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K, kBK, kBM);
+  if (e != cudaSuccess) return e;
+  e = make_tmap_bf16_2d(&tb, a.W, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K, kBK, kBN);
+  if (e != cudaSuccess) return e;
+  const int smem = (int)sizeof(GemmSmem) + 1024;
+  e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const int tiles = ((a.M + kBM - 1) / kBM) * ((a.N + kBN - 1) / kBN);
+  GemmParams prm{a.M, a.N, a.K, a.bias, a.act, a.scale, a.residual, a.out, a.err};
+  gemm_kernel<<<min(num_sms, tiles), 192, smem, st>>>(ta, tb, prm);
+  return cudaGetLastError();
+}
+
+}  // namespace vp

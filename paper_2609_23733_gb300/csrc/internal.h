@@ -1,0 +1,115 @@
+// Internal launchers and workspace layout of the sm_103a library (not part of the ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "vp.h"
+
+namespace vp {
+
+constexpr int kHeadDim = 64;
+constexpr int kHidden = 64;
+constexpr int kMaxHeads = 32;
+constexpr int kQTile = 128;          // query rows per full-attention work item
+constexpr int kPoolSplitMax = 64;    // CTAs per head in the pooling sweep
+constexpr int kKeySplitMax = 64;     // CTAs per head in the key sweep
+constexpr int kPoolPartial = 2 + kHeadDim;          // (max, sum, sum p q[64])
+constexpr int kKeyPartial = 2 + 2 * kHeadDim;       // (max, sum, sum p v[64], sum v[64])
+
+// Router scratch carved from the caller's workspace (all device pointers).
+struct RouterScratch {
+  unsigned int* err;            // device error word (first 256 bytes of the workspace)
+  unsigned int* counters;       // [2 * kMaxHeads + 2] last-CTA counters, zeroed per call
+  float* pool_part;             // [H][kPoolSplitMax][kPoolPartial]
+  float* key_part;              // [H][kKeySplitMax][kKeyPartial]
+  float* q_pool;                // [H][64]
+  float* key_stats;             // [H][2] (global max of scaled logits, sum of exp)
+  float* s;                     // [H]
+  int32_t* modes;               // [H]
+  float* ctx;                   // [H][64]
+  float* mean_v;                // [H][64]
+  int32_t* head_ids;            // [H]
+  int32_t* offsets;             // [4]
+};
+
+size_t router_scratch_bytes(int H);
+RouterScratch carve_router_scratch(void* ws, int H);
+
+struct RouterArgs {
+  int N, H;
+  float tau_low, tau_high;
+  const __nv_bfloat16* qkv;
+  const __nv_bfloat16* W;
+  const __nv_bfloat16* U;
+  const __nv_bfloat16* w;
+  const float* bW;
+  const float* bU;
+  const float* beta;
+  const int32_t* force_modes;
+  // Outputs (NULL = do not copy out); the scratch copies are always written.
+  float* s_out;
+  int32_t* modes_out;
+  float* q_pool_out;
+  float* ctx_out;
+  float* mean_v_out;
+  float* r_out;
+};
+
+cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_sms,
+                          cudaStream_t st);
+cudaError_t launch_bin_heads(int H, int N, const int32_t* modes, int32_t* head_ids,
+                             int32_t* offsets, int32_t* work, int32_t* n_work, cudaStream_t st);
+
+struct SurrogateArgs {
+  const __nv_bfloat16* g1_w; const float* g1_b;
+  const __nv_bfloat16* g2_w; const float* g2_b;
+  const __nv_bfloat16* d1_w; const float* d1_b;
+  const __nv_bfloat16* d2_w; const float* d2_b;
+};
+
+struct HeadAttnArgs {
+  int N, H;
+  const __nv_bfloat16* qkv;
+  const int32_t* head_ids;
+  const int32_t* offsets;
+  const float* ctx;
+  const float* mean_v;
+  SurrogateArgs sw;
+  __nv_bfloat16* y;
+  unsigned int* err;
+};
+
+cudaError_t launch_mean_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_surrogate_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+
+struct LinearArgs {
+  int M, N, K;
+  const __nv_bfloat16* A;
+  const __nv_bfloat16* W;
+  const float* bias;
+  int act;
+  const float* scale;
+  const __nv_bfloat16* residual;
+  __nv_bfloat16* out;
+  unsigned int* err;   // may be NULL (vp_linear has no workspace): a private word is used
+};
+cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st);
+
+cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float* g,
+                              const float* b, float eps, __nv_bfloat16* out, cudaStream_t st);
+
+// Host-side TMA descriptor creation (driver entry point fetched at run time).
+// 2-D bf16 tensor [rows][cols] with a row pitch of `pitch_elems`, box of box_cols x box_rows,
+// 128-byte swizzle, zero fill out of bounds.
+cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
+                              uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows);
+
+int device_sm_count();
+bool device_is_sm103();
+
+}  // namespace vp
