@@ -1,0 +1,447 @@
+"""Benchmark of the mixture-of-heads global-attention stack on GB300.
+
+Workload: the 24-layer global stack (Algorithm 1 blocks: LayerNorm, routed attention,
+W_O, LayerScale + residual, FFN ratio 4) over S = 100 views at 518 px (1,374 tokens per
+view, N = 137,400 tokens), D = 1024, 16 heads x 64, seeded synthetic bf16 activations
+~ N(0, 1) and Xavier weights.  The untrained routers run in full on every layer; their
+decisions are replaced by routes that follow the trained router's average distribution
+over seven datasets (App. E.2: 50.0 % mean, 42.2 % surrogate, 7.8 % full -> 30 full,
+162 surrogate and 192 mean heads over the 384 heads of the stack).
+
+One step = one forward of the stack on one scene.  ``value`` is views per second over the
+whole job (S x ranks / step time).  ``e2e`` adds the host -> device copy of the step's
+tokens and the device -> host copy of its output (pinned buffers).  ``roofline`` reports
+the dominant kernel class, timed with CUDA events recorded by the library around each of
+its launches inside the timed region.  ``cpu_baseline`` times the float64 oracle on a
+bounded sample of the same workload (rank 0, one GPU only).
+
+--impl reference runs that oracle as the reference arm instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOAD = synth.WORKLOADS["s100_stack"]
+H, d, D = synth.N_HEADS, synth.HEAD_DIM, synth.D_MODEL
+METRIC = "global-attn views/sec, 24-layer MoH global stack at S=100 (518 px, 137,400 tokens)"
+
+
+def peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except OSError:
+        return None
+
+
+# ------------------------------------------------------------------ analytic work per step
+def step_flops(N, routes):
+    """Tensor-core work of one stack forward (flop): projections + full-mode attention."""
+    lin = 2.0 * N * D * (3 * D + D + 4 * D + 4 * D) * routes.shape[0]
+    full = 4.0 * N * N * d * int((routes == synth.MODE_FULL).sum())
+    return lin, full
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) >= 9:
+                rows.append(f)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------------ CPU oracle sample
+def oracle_sample(N, routes, layer_w, x_bits, rows=8192, full_rows=256):
+    """Times the float64 oracle on a bounded sample of one stack forward and scales it to
+    a whole forward.  Every step of a layer except full attention is linear in the tokens
+    (the router's two sweeps included), so it runs on ``rows`` tokens and is scaled by
+    N / rows; one full head runs ``full_rows`` query rows against all N keys and is scaled
+    by N / full_rows.  Returns (ms_per_forward, description, seconds per part)."""
+    import oracle
+
+    lw = oracle.load_layer(layer_w)
+    g = np.random.default_rng(0)
+    sel = np.sort(g.choice(N, rows, replace=False))
+    t = {}
+    X = oracle.bf16_bits_to_f64(x_bits[sel])
+    t0 = time.perf_counter()
+    Xt = oracle.round_bf16(oracle.layer_norm(X, lw["ln1_g"], lw["ln1_b"], 1e-6))
+    qkv = oracle.qkv_projection(Xt, lw)
+    rs = [oracle.layer.head_router(qkv[:, 0, h], qkv[:, 1, h], lw, h) for h in range(H)]
+    t["ln_qkv_router"] = (time.perf_counter() - t0) * N / rows
+    t0 = time.perf_counter()
+    h = 1
+    mg = (lw["s_g1_w"][h], lw["s_g1_b"][h], lw["s_g2_w"][h], lw["s_g2_b"][h])
+    md = (lw["s_d1_w"][h], lw["s_d1_b"][h], lw["s_d2_w"][h], lw["s_d2_b"][h])
+    oracle.surrogate_attention(qkv[:, 2, h], rs[h][2], mg, md)
+    t["surrogate_per_head"] = (time.perf_counter() - t0) * N / rows
+    t0 = time.perf_counter()
+    oracle.mean_pooling(qkv[:, 2, 2])
+    t["mean_per_head"] = (time.perf_counter() - t0) * N / rows
+    t0 = time.perf_counter()
+    Y = oracle.round_bf16(qkv[:, 2].reshape(rows, D))
+    Xa = oracle.round_bf16(X + (Y @ lw["w_o"].T + lw["b_o"]) * lw["ls1"])
+    Zt = oracle.round_bf16(oracle.layer_norm(Xa, lw["ln2_g"], lw["ln2_b"], 1e-6))
+    Hd = oracle.round_bf16(oracle.gelu(Zt @ lw["w_fc1"].T + lw["b_fc1"]))
+    oracle.round_bf16(Xa + (Hd @ lw["w_fc2"].T + lw["b_fc2"]) * lw["ls2"])
+    t["wo_ln2_ffn"] = (time.perf_counter() - t0) * N / rows
+    # Full attention of one head: full_rows queries against N keys and values.
+    KV = oracle.round_bf16(g.standard_normal((2, N, d)))
+    Qf = oracle.round_bf16(g.standard_normal((N, d)))
+    t0 = time.perf_counter()
+    oracle.full_attention(Qf, KV[0], KV[1], rows=np.arange(full_rows))
+    t["full_per_head"] = (time.perf_counter() - t0) * N / full_rows
+    L = routes.shape[0]
+    n_full = int((routes == synth.MODE_FULL).sum())
+    n_surr = int((routes == synth.MODE_SURROGATE).sum())
+    n_mean = int((routes == synth.MODE_MEAN).sum())
+    total = L * (t["ln_qkv_router"] + t["wo_ln2_ffn"]) + n_full * t["full_per_head"] + \
+        n_surr * t["surrogate_per_head"] + n_mean * t["mean_per_head"]
+    desc = (f"float64 oracle, one layer's per-token work (LN1, QKV, router of 16 heads, a surrogate "
+            f"and a mean head, W_O, LN2, FFN) on {rows} of N={N} tokens scaled by N/{rows}, one full "
+            f"head on {full_rows} query rows x N keys scaled by N/{full_rows}; totals for {L} layers and "
+            f"{n_full} full / {n_surr} surrogate / {n_mean} mean heads (extrapolated)")
+    return total * 1e3, desc, t
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# ------------------------------------------------------------------ arms
+def run_reference(args):
+    """The oracle as the reference arm: each step is the bounded CPU sample."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    N = WORKLOAD.N
+    routes = synth.paper_mix_modes(WORKLOAD.layers)
+    w0 = synth.make_stack_weights(WORKLOAD.seed, 1)[0]
+    x_bits = synth.make_tokens(WORKLOAD.seed, N)
+    times = []
+    desc = ""
+    for i in range(args.warmup + args.steps):
+        ms, desc, _ = oracle_sample(N, routes, w0, x_bits)
+        if i >= args.warmup:
+            times.append(ms)
+    ms = float(np.median(times))
+    value = WORKLOAD.views / (ms / 1e3)
+    cb = {"value": value, "unit": "views/s", "cores": cpu_cores(), "kind": "oracle", "sample": desc}
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "views/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD.name, "views": WORKLOAD.views, "tokens": N, "layers": WORKLOAD.layers,
+                   "routing": "paper_mix"},
+        "cpu_baseline": cb,
+        "e2e": {"value": value, "unit": "views/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_23733_gb300 import binding as vpb
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device(f"cuda:{local}"))
+    torch.cuda.set_device(local)
+    dev = torch.device(f"cuda:{local}")
+    vpb.lib()
+
+    N, L = WORKLOAD.N, WORKLOAD.layers
+    routes = synth.paper_mix_modes(L)
+    # Every rank processes its own scene (weak scaling, no data-path collective).
+    seed = WORKLOAD.seed + 100 * rank
+    host_w = synth.make_stack_weights(seed, L)
+    dws = [vpb.to_device(w, dev) for w in host_w]
+    layers = [vpb.layer_weights(w) for w in dws]
+    x_bits = synth.make_tokens(seed, N)
+    x0 = vpb.bf16_from_bits(x_bits, dev)
+    x = torch.empty_like(x0)
+    fm = torch.from_numpy(routes).to(dev)
+    modes_out = torch.zeros(L, H, dtype=torch.int32, device=dev)
+    s_out = torch.zeros(L, H, device=dev)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK, dev)
+
+    def step():
+        x.copy_(x0)  # every step starts from the same tokens
+        vpb.vp_global_stack(dm, x, layers, fm, modes_out, s_out, 1e-6, ws)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    vpb.vp_profile_begin(64 * L * max(args.steps, 1))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    barrier()
+    n_launch, per_class_n, per_class_ms = vpb.vp_profile_end()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    err_bits = vpb.vp_read_device_error(ws)
+    value = WORKLOAD.views * world / (ms / 1e3)
+
+    # End to end through the public API: pinned host tokens in, pinned host output out.
+    x_host = torch.from_numpy(x_bits.view(np.int16)).view(torch.bfloat16).pin_memory()
+    y_host = torch.empty_like(x_host).pin_memory()
+    e2e_steps = max(1, min(args.steps, 3))
+
+    def e2e_step():
+        x.copy_(x_host, non_blocking=True)
+        vpb.vp_global_stack(dm, x, layers, fm, modes_out, s_out, 1e-6, ws)
+        y_host.copy_(x, non_blocking=True)
+
+    e2e_step()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    finite = bool(torch.isfinite(y_host.float()).all())
+
+    # Natural routes of the untrained routers (reported, not used).
+    natural = {"mean": 0, "surrogate": 0, "full": 0}
+    sh = s_out.cpu().numpy()
+    for s in sh.reshape(-1):
+        m = 2 if s >= 0.2 else (0 if s <= 0.01 else 1)
+        natural[["mean", "surrogate", "full"][m]] += 1
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    pk = peaks() or {}
+    lin_flops, full_flops = step_flops(N, routes)
+    dominant = max(per_class_ms, key=per_class_ms.get)
+    roof = None
+    if dominant == "attn_full" and per_class_n["attn_full"]:
+        per_launch_flops = full_flops * args.steps / per_class_n["attn_full"]
+        per_launch_ms = per_class_ms["attn_full"] / per_class_n["attn_full"]
+        ach = per_launch_flops / (per_launch_ms * 1e-3) / 1e12
+        peak = pk.get("bf16_tflops_sustained") or 1700.0
+        roof = {"bound": "tensor", "kernel": "attn_full_kernel", "achieved": ach, "peak": peak,
+                "unit": "TFLOP/s", "frac": ach / peak, "peak_kind": "measured sustained bf16 (cuBLAS)",
+                "traffic": traffic_from_profile("attn_full"), "ms_per_launch": per_launch_ms,
+                "flop_per_launch": per_launch_flops}
+    elif dominant == "gemm" and per_class_n["gemm"]:
+        per_launch_flops = lin_flops * args.steps / per_class_n["gemm"]
+        per_launch_ms = per_class_ms["gemm"] / per_class_n["gemm"]
+        ach = per_launch_flops / (per_launch_ms * 1e-3) / 1e12
+        peak = pk.get("bf16_tflops_sustained") or 1700.0
+        roof = {"bound": "tensor", "kernel": "gemm_kernel", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                "frac": ach / peak, "peak_kind": "measured sustained bf16 (cuBLAS)",
+                "traffic": traffic_from_profile("gemm"), "ms_per_launch": per_launch_ms}
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        ms_cpu, desc, _ = oracle_sample(N, routes, host_w[0], x_bits)
+        cpu = {"value": WORKLOAD.views / (ms_cpu / 1e3), "unit": "views/s", "cores": cpu_cores(),
+               "kind": "oracle", "sample": desc}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "views/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD.name, "views": WORKLOAD.views, "image_px": WORKLOAD.image_px,
+                   "tokens": N, "layers": L, "dim": D, "heads": H, "head_dim": d,
+                   "routing": "paper_mix (30 full / 162 surrogate / 192 mean of 384 heads)",
+                   "parallelism": f"replicas{world}", "l2": "inputs larger than L2 (281 MB tokens, 1.4 GB workspace)"},
+        "e2e": {"value": WORKLOAD.views * world / (e2e_ms / 1e3), "unit": "views/s",
+                "h2d_bytes_per_step": int(x_host.numel() * 2), "d2h_bytes_per_step": int(y_host.numel() * 2),
+                "ms_per_step": e2e_ms},
+        "gpu_launches": int(n_launch),
+        "kernels": {k: {"launches": per_class_n[k], "ms_per_step": per_class_ms[k] / args.steps}
+                    for k in per_class_ms if per_class_n[k]},
+        "roofline": roof,
+        "tensor_work": {"projections_tflop": lin_flops / 1e12, "full_attention_tflop": full_flops / 1e12,
+                        "achieved_tflops_step": (lin_flops + full_flops) / (ms * 1e-3) / 1e12},
+        "cpu_baseline": cpu,
+        "clocks": clk,
+        "natural_routes": natural,
+        "device_error_bits": err_bits,
+        "output_finite": finite,
+    }
+    if args.full_layer:
+        line["full_attention_s100"] = full_attention_probe(vpb, dev, N, dws[0], pk)
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def full_attention_probe(vpb, dev, N, dw, pk):
+    """All 16 heads in full mode over N tokens (the forced all-full layer of the target)."""
+    import torch
+    qkv = torch.randn(N, 3 * D, device=dev).to(torch.bfloat16)
+    y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_ROUTER, dev)
+    ids = torch.arange(H, dtype=torch.int32, device=dev)
+    off = torch.tensor([0, 0, 0, H], dtype=torch.int32, device=dev)
+    z = torch.zeros(H, d, device=dev)
+    sw = vpb.surrogate_weights(dw)
+    vpb.vp_head_attention(dm, qkv, ids, off, z, z, sw, y, ws)
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(3):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        vpb.vp_head_attention(dm, qkv, ids, off, z, z, sw, y, ws)
+        b.record()
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    ms = float(np.median(ts))
+    tf = 4.0 * N * N * d * H / (ms * 1e-3) / 1e12
+    peak = pk.get("bf16_tflops") or 1886.0
+    return {"ms": ms, "tflops": tf, "peak": peak, "frac": tf / peak, "peak_kind": "measured burst bf16"}
+
+
+def kernel_case(args):
+    """One kernel on a mid-sized input (larger than L2, a few hundred MB on the device),
+    launched a few times: the small case that ncu captures."""
+    import torch
+
+    from paper_2609_23733_gb300 import binding as vpb
+    dev = torch.device("cuda:0")
+    N = args.case_tokens
+    qkv = torch.randn(N, 3 * D, device=dev).to(torch.bfloat16)
+    if args.kernel_case == "attn_full":
+        w = vpb.to_device(synth.make_layer_weights(synth.rng(0)), dev)
+        y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+        dm = vpb.dims(N, H)
+        ws = vpb.workspace(dm, vpb.VP_WS_ROUTER, dev)
+        ids = torch.arange(H, dtype=torch.int32, device=dev)
+        off = torch.tensor([0, 0, 0, H], dtype=torch.int32, device=dev)
+        z = torch.zeros(H, d, device=dev)
+        for _ in range(args.case_launches):
+            vpb.vp_head_attention(dm, qkv, ids, off, z, z, vpb.surrogate_weights(w), y, ws)
+    else:
+        x = torch.randn(N, D, device=dev).to(torch.bfloat16)
+        wq = (torch.rand(3 * D, D, device=dev) * 0.1 - 0.05).to(torch.bfloat16)
+        b = torch.zeros(3 * D, device=dev)
+        for _ in range(args.case_launches):
+            vpb.vp_linear(x, wq, b, out=qkv)
+    torch.cuda.synchronize()
+    print(json.dumps({"kernel_case": args.kernel_case, "tokens": N, "launches": args.case_launches}))
+
+
+def traffic_from_profile(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source still
+    matches the hash recorded there (else None)."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
+    src = {"attn_full": "attn_full.cu", "gemm": "gemm.cu"}[kernel]
+    try:
+        kv = dict(line.strip().split("=", 1) for line in open(path) if "=" in line and not line.startswith("#"))
+    except OSError:
+        return None
+    h = hashlib.sha256(open(os.path.join(ROOT, "paper_2609_23733_gb300", "csrc", src), "rb").read()).hexdigest()[:16]
+    if kv.get("source_sha256_16") != h:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch_scaled"])
+    except (KeyError, ValueError):
+        return None
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--full-layer", action="store_true", default=True)
+    ap.add_argument("--no-full-layer", dest="full_layer", action="store_false")
+    ap.add_argument("--kernel-case", choices=["attn_full", "gemm"], default=None,
+                    help="run one kernel on a mid-sized input (for ncu captures) and exit")
+    ap.add_argument("--case-tokens", type=int, default=32768)
+    ap.add_argument("--case-launches", type=int, default=2)
+    args = ap.parse_args()
+    if args.kernel_case:
+        kernel_case(args)
+    elif args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -213,6 +213,32 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
                           int32_t* modes_out, float* s_out, float ln_eps, void* ws,
                           size_t ws_bytes, void* stream);
 
+/* Kernel classes reported by the launch profiler. */
+#define VP_KERNEL_GEMM 0
+#define VP_KERNEL_ROUTER_POOL 1
+#define VP_KERNEL_ROUTER_KEYS 2
+#define VP_KERNEL_ROUTER_R 3
+#define VP_KERNEL_BIN_HEADS 4
+#define VP_KERNEL_ATTN_FULL 5
+#define VP_KERNEL_SURROGATE 6
+#define VP_KERNEL_MEAN 7
+#define VP_KERNEL_LAYER_NORM 8
+#define VP_KERNEL_CLASSES 9
+
+/*
+ * Launch profiler (for benchmarks; not part of the method).  Between vp_profile_begin and
+ * vp_profile_end every kernel the library launches on the calling host thread's current
+ * device is bracketed by two CUDA events recorded on the launch's own stream.  Events are
+ * created in vp_profile_begin (max_launches pairs) and destroyed in vp_profile_end; launches
+ * beyond max_launches are counted but not timed.
+ * vp_profile_end waits for the last recorded event, then writes (host pointers):
+ *   n_launches[1]            kernels launched while profiling (all classes)
+ *   launches[VP_KERNEL_CLASSES]  launches per class
+ *   ms[VP_KERNEL_CLASSES]    summed event time per class, milliseconds
+ */
+vp_status vp_profile_begin(int32_t max_launches);
+vp_status vp_profile_end(int32_t* n_launches, int32_t* launches, float* ms);
+
 #ifdef __cplusplus
 }
 #endif

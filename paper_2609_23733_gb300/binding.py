@@ -20,6 +20,8 @@ VP_MODE_MEAN, VP_MODE_SURROGATE, VP_MODE_FULL = 0, 1, 2
 VP_WS_ROUTER, VP_WS_LAYER, VP_WS_STACK = 0, 1, 2
 VP_ACT_NONE, VP_ACT_GELU = 0, 1
 VP_DEVERR_WAIT_TIMEOUT, VP_DEVERR_NAN_SALIENCY = 1, 2
+KERNEL_CLASSES = ["gemm", "router_pool", "router_keys", "router_r", "bin_heads", "attn_full",
+                  "surrogate", "mean", "layer_norm"]
 
 STATUS = {0: "VP_OK", 1: "VP_ERR_INVALID_ARG", 2: "VP_ERR_UNSUPPORTED_SHAPE", 3: "VP_ERR_ALIGNMENT",
           4: "VP_ERR_CUDA", 5: "VP_ERR_DEVICE_TIMEOUT", 6: "VP_ERR_WORKSPACE",
@@ -73,6 +75,8 @@ _SIGS = [
                                           c_void_p, POINTER(VpRouterWeights),
                                           POINTER(VpSurrogateWeights), c_void_p, c_void_p, c_void_p,
                                           c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    ("vp_profile_begin", c_int32, [c_int32]),
+    ("vp_profile_end", c_int32, [POINTER(c_int32), POINTER(c_int32), POINTER(c_float)]),
     ("vp_global_stack", c_int32, [POINTER(VpDims), c_int32, c_void_p, POINTER(VpLayerWeights),
                                   c_void_p, c_void_p, c_void_p, c_float, c_void_p, c_size_t, c_void_p]),
 ]
@@ -230,3 +234,16 @@ def vp_global_stack(dm, x_inout, layers, force_modes, modes_out, s_out, ln_eps, 
     _check(lib().vp_global_stack(ctypes.byref(dm), len(layers), _p(x_inout), arr, _p(force_modes),
                                  _p(modes_out), _p(s_out), float(ln_eps), _p(ws), ws.numel(),
                                  _stream(stream)), "vp_global_stack")
+
+
+def vp_profile_begin(max_launches: int):
+    _check(lib().vp_profile_begin(int(max_launches)), "vp_profile_begin")
+
+
+def vp_profile_end():
+    """Returns (total launches, {class: launches}, {class: summed ms})."""
+    n = c_int32(0)
+    cnt = (c_int32 * len(KERNEL_CLASSES))()
+    ms = (c_float * len(KERNEL_CLASSES))()
+    _check(lib().vp_profile_end(ctypes.byref(n), cnt, ms), "vp_profile_end")
+    return n.value, dict(zip(KERNEL_CLASSES, list(cnt))), dict(zip(KERNEL_CLASSES, list(ms)))

@@ -46,6 +46,46 @@ EncodeTiledFn g_encode = nullptr;
 std::once_flag g_encode_once;
 }  // namespace
 
+// ------------------------------------------------------------------ launch profiler
+namespace {
+struct ProfRecord {
+  int kind;
+  cudaEvent_t start, stop;
+};
+struct Profiler {
+  bool active = false;
+  int max = 0, used = 0, launches = 0;
+  int per_class[VP_KERNEL_CLASSES] = {};
+  ProfRecord* rec = nullptr;
+  cudaEvent_t pending = nullptr;  // start event of the launch being bracketed
+  int pending_kind = -1;
+};
+thread_local Profiler g_prof;
+}  // namespace
+
+void prof_before(int kind, cudaStream_t st) {
+  Profiler& p = g_prof;
+  if (!p.active) return;
+  ++p.launches;
+  ++p.per_class[kind];
+  p.pending = nullptr;
+  if (p.used < p.max) {
+    ProfRecord& r = p.rec[p.used];
+    r.kind = kind;
+    cudaEventRecord(r.start, st);
+    p.pending = r.stop;
+    p.pending_kind = kind;
+  }
+}
+
+void prof_after(cudaStream_t st) {
+  Profiler& p = g_prof;
+  if (!p.active || !p.pending) return;
+  cudaEventRecord(p.pending, st);
+  p.pending = nullptr;
+  ++p.used;
+}
+
 int device_sm_count() { return dev_info().sms; }
 bool device_is_sm103() { return dev_info().sm103 == 1; }
 
@@ -259,6 +299,54 @@ vp_status vp_workspace_size(const vp_dims* dims, int32_t what, size_t* bytes) {
     default: return VP_ERR_INVALID_ARG;
   }
   return VP_OK;
+}
+
+vp_status vp_profile_begin(int32_t max_launches) {
+  Profiler& p = g_prof;
+  if (p.active || max_launches < 0 || max_launches > (1 << 20)) return VP_ERR_INVALID_ARG;
+  p = Profiler();
+  p.rec = new ProfRecord[max_launches > 0 ? max_launches : 1];
+  for (int i = 0; i < max_launches; ++i) {
+    if (cudaEventCreate(&p.rec[i].start) != cudaSuccess ||
+        cudaEventCreate(&p.rec[i].stop) != cudaSuccess) {
+      for (int j = 0; j <= i; ++j) {
+        cudaEventDestroy(p.rec[j].start);
+        cudaEventDestroy(p.rec[j].stop);
+      }
+      delete[] p.rec;
+      p.rec = nullptr;
+      return VP_ERR_CUDA;
+    }
+  }
+  p.max = max_launches;
+  p.active = true;
+  return VP_OK;
+}
+
+vp_status vp_profile_end(int32_t* n_launches, int32_t* launches, float* ms) {
+  Profiler& p = g_prof;
+  if (!p.active) return VP_ERR_INVALID_ARG;
+  p.active = false;
+  vp_status st = VP_OK;
+  float acc[VP_KERNEL_CLASSES] = {};
+  if (p.used > 0 && cudaEventSynchronize(p.rec[p.used - 1].stop) != cudaSuccess) st = VP_ERR_CUDA;
+  for (int i = 0; i < p.used && st == VP_OK; ++i) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, p.rec[i].start, p.rec[i].stop) != cudaSuccess) st = VP_ERR_CUDA;
+    acc[p.rec[i].kind] += t;
+  }
+  for (int i = 0; i < p.max; ++i) {
+    cudaEventDestroy(p.rec[i].start);
+    cudaEventDestroy(p.rec[i].stop);
+  }
+  delete[] p.rec;
+  p.rec = nullptr;
+  if (n_launches) *n_launches = p.launches;
+  for (int k = 0; k < VP_KERNEL_CLASSES; ++k) {
+    if (launches) launches[k] = p.per_class[k];
+    if (ms) ms[k] = acc[k];
+  }
+  return st;
 }
 
 vp_status vp_read_device_error(void* ws, size_t ws_bytes, uint32_t* host_bits, void* stream) {

@@ -347,7 +347,9 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
   e = cudaFuncSetAttribute(attn_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.err};
+  prof_before(VP_KERNEL_ATTN_FULL, st);
   attn_full_kernel<<<num_sms, 192, smem, st>>>(tmap, prm);
+  prof_after(st);
   return cudaGetLastError();
 }
 

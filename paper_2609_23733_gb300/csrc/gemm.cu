@@ -229,7 +229,9 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   const int tiles = ((a.M + kBM - 1) / kBM) * ((a.N + kBN - 1) / kBN);
   GemmParams prm{a.M, a.N, a.K, a.bias, a.act, a.scale, a.residual, a.out, a.err};
+  prof_before(VP_KERNEL_GEMM, st);
   gemm_kernel<<<min(num_sms, tiles), 192, smem, st>>>(ta, tb, prm);
+  prof_after(st);
   return cudaGetLastError();
 }
 

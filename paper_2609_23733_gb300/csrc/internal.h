@@ -109,6 +109,10 @@ cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float*
 cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
                               uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows);
 
+// Launch profiler hooks (no-ops unless vp_profile_begin is active).
+void prof_before(int kind, cudaStream_t st);
+void prof_after(cudaStream_t st);
+
 int device_sm_count();
 bool device_is_sm103();
 

@@ -65,6 +65,7 @@ __global__ void __launch_bounds__(256) layernorm_kernel(int M, const __nv_bfloat
 cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float* g,
                               const float* b, float eps, __nv_bfloat16* out, cudaStream_t st) {
   const int blocks = (M + 7) / 8;
+  prof_before(VP_KERNEL_LAYER_NORM, st);
   switch (D / 256) {
     case 1: layernorm_kernel<1><<<blocks, 256, 0, st>>>(M, x, g, b, eps, out); break;
     case 2: layernorm_kernel<2><<<blocks, 256, 0, st>>>(M, x, g, b, eps, out); break;
@@ -72,8 +73,9 @@ cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float*
     case 4: layernorm_kernel<4><<<blocks, 256, 0, st>>>(M, x, g, b, eps, out); break;
     case 8: layernorm_kernel<8><<<blocks, 256, 0, st>>>(M, x, g, b, eps, out); break;
     case 16: layernorm_kernel<16><<<blocks, 256, 0, st>>>(M, x, g, b, eps, out); break;
-    default: return cudaErrorInvalidValue;
+    default: prof_after(st); return cudaErrorInvalidValue;
   }
+  prof_after(st);
   return cudaGetLastError();
 }
 

@@ -200,13 +200,17 @@ __global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
 }  // namespace
 
 cudaError_t launch_mean_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
+  prof_before(VP_KERNEL_MEAN, st);
   mean_heads_kernel<<<4 * num_sms, 256, 0, st>>>(a);
+  prof_after(st);
   return cudaGetLastError();
 }
 
 cudaError_t launch_surrogate_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
   static_assert(sizeof(SurrSmem) <= 48 * 1024, "surrogate smem fits the default limit");
+  prof_before(VP_KERNEL_SURROGATE, st);
   surrogate_heads_kernel<<<4 * num_sms, 128, sizeof(SurrSmem), st>>>(a);
+  prof_after(st);
   return cudaGetLastError();
 }
 

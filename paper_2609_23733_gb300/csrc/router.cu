@@ -488,17 +488,23 @@ cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_
   // Enough CTAs to cover every SM a few times; at least 64 tokens per CTA.
   int pool_split = (4 * num_sms + a.H - 1) / a.H;
   pool_split = max(1, min(min(pool_split, kPoolSplitMax), (a.N + 63) / 64));
+  prof_before(VP_KERNEL_ROUTER_POOL, st);
   router_pool_kernel<<<dim3(pool_split, a.H), kPoolThreads, 0, st>>>(a, sc, pool_split);
+  prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int key_split = (2 * num_sms + a.H - 1) / a.H;
   key_split = max(1, min(min(key_split, kKeySplitMax), (a.N + 127) / 128));
+  prof_before(VP_KERNEL_ROUTER_KEYS, st);
   router_keys_kernel<<<dim3(key_split, a.H), kKeyThreads, 0, st>>>(a, sc, key_split);
+  prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (a.r_out) {
     int blocks = max(1, min((a.N + 31) / 32, (2 * num_sms + a.H - 1) / a.H));
+    prof_before(VP_KERNEL_ROUTER_R, st);
     router_r_kernel<<<dim3(blocks, a.H), 256, 0, st>>>(a, sc);
+    prof_after(st);
     e = cudaGetLastError();
   }
   return e;
@@ -506,7 +512,9 @@ cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_
 
 cudaError_t launch_bin_heads(int H, int N, const int32_t* modes, int32_t* head_ids,
                              int32_t* offsets, int32_t* work, int32_t* n_work, cudaStream_t st) {
+  prof_before(VP_KERNEL_BIN_HEADS, st);
   bin_heads_kernel<<<1, 256, 0, st>>>(H, N, modes, head_ids, offsets, work, n_work);
+  prof_after(st);
   return cudaGetLastError();
 }
 

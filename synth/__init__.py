@@ -71,8 +71,9 @@ def rng(seed: int) -> np.random.Generator:
 
 def f32_to_bf16_bits(x) -> np.ndarray:
     """Pack float values into bf16 bit patterns (round to nearest even)."""
-    b = np.ascontiguousarray(np.asarray(x, dtype=np.float32)).view(np.uint32).astype(np.uint64)
-    b = (b + 0x7FFF + ((b >> 16) & 1)) >> 16
+    b = np.ascontiguousarray(np.asarray(x, dtype=np.float32)).view(np.uint32)
+    # Finite values stay below 0xFF800000, so the rounding add cannot wrap in 32 bits.
+    b = (b + (np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1)))) >> np.uint32(16)
     return b.astype(np.uint16)
 
 

@@ -15,14 +15,22 @@ MEAN_ABS = 2e-3
 GUARD = 1e-3
 
 
-def compare(got, want, max_abs=MAX_ABS, mean_abs=MEAN_ABS, what=""):
+# Both sides round a stored bf16 value independently; a value within rounding noise of a
+# rounding boundary may land one bf16 step (2^-7 relative at most) apart.  ``rel`` adds that
+# step for large-magnitude outputs (the residual stream), where one step exceeds MAX_ABS.
+BF16_STEP = 2.0 ** -7
+
+
+def compare(got, want, max_abs=MAX_ABS, mean_abs=MEAN_ABS, rel=0.0, what=""):
     got = np.asarray(got, np.float64)
     want = np.asarray(want, np.float64)
     assert got.shape == want.shape, (what, got.shape, want.shape)
     assert np.all(np.isfinite(got)), f"{what}: non-finite values"
     err = np.abs(got - want)
+    excess = err - (max_abs + rel * np.abs(want))
     mx, mn = float(err.max(initial=0.0)), float(err.mean()) if err.size else 0.0
-    assert mx <= max_abs and mn <= mean_abs, f"{what}: max-abs {mx:.3e} mean-abs {mn:.3e}"
+    assert float(excess.max(initial=-1.0)) <= 0 and mn <= mean_abs, \
+        f"{what}: max-abs {mx:.3e} mean-abs {mn:.3e} (worst excess {float(excess.max(initial=0)):.3e})"
     return mx, mn
 
 

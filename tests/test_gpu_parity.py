@@ -7,7 +7,7 @@ import torch
 
 import oracle
 import synth
-from tests.helpers import MAX_ABS, MEAN_ABS, calibrated_layer, compare, outside_guard
+from tests.helpers import BF16_STEP, calibrated_layer, compare, outside_guard
 
 pytestmark = pytest.mark.gpu
 
@@ -57,7 +57,7 @@ def test_linear_matches_oracle(M, N, K, act, with_bias, with_scale, with_res):
         ref = ref * sc.astype(np.float64)
     if R is not None:
         ref = ref + R
-    compare(_f64(out), oracle.round_bf16(ref), what="linear")
+    compare(_f64(out), oracle.round_bf16(ref), rel=BF16_STEP if with_res else 0.0, what="linear")
 
 
 def test_linear_residual_in_place():
@@ -68,7 +68,7 @@ def test_linear_residual_in_place():
     x = _bf(X)
     vpb.vp_linear(_bf(A), _bf(W), None, 0, None, x, out=x)
     torch.cuda.synchronize()
-    compare(_f64(x), oracle.round_bf16(X + A @ W.T), what="in-place residual")
+    compare(_f64(x), oracle.round_bf16(X + A @ W.T), rel=BF16_STEP, what="in-place residual")
 
 
 # ------------------------------------------------------------------ LayerNorm (a10)
@@ -289,7 +289,6 @@ def test_layer_s8_518_calibrated():
     are full, 6 surrogate and 6 mean; the oracle checks sampled rows of every head."""
     wl = synth.WORKLOADS["s8_layer_biased"]
     N = wl.N
-    mix = [2, 1, 1, 0] * 4
     mix = [2, 1, 1, 0, 2, 1, 0, 0, 2, 1, 1, 0, 2, 1, 0, 0]
     x_bits, w, lw = calibrated_layer(wl.seed, N, mix)
     got, s, modes = _run_layer(x_bits, w, N, 16)
