@@ -51,7 +51,9 @@ typedef enum vp_status {
   VP_ERR_CUDA = 4,               /* a CUDA call or launch failed */
   VP_ERR_DEVICE_TIMEOUT = 5,     /* a kernel gave up waiting (see device error word) */
   VP_ERR_WORKSPACE = 6,          /* workspace missing or smaller than vp_workspace_size */
-  VP_ERR_UNSUPPORTED_DEVICE = 7  /* the current device is not sm_103 */
+  VP_ERR_UNSUPPORTED_DEVICE = 7, /* the current device is not sm_103 */
+  VP_ERR_STATIC_SCRATCH = 8      /* vp_router_noalloc: the call needs more scratch than its
+                                    fixed buffer holds */
 } vp_status;
 
 /* Routed computation modes, §4.2 routing equation. */
@@ -212,6 +214,29 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
                           const vp_layer_weights* layers, const int32_t* force_modes,
                           int32_t* modes_out, float* s_out, float ln_eps, void* ws,
                           size_t ws_bytes, void* stream);
+
+/*
+ * vp_router_noalloc -- vp_router without a workspace, for callers that cannot allocate
+ * device memory when they call the router (for example a plug-in inside a host framework
+ * whose memory pool already reserves the GPU's memory and forbids raw cudaMalloc, or a
+ * service that must not allocate once it is running).  The paper has no counterpart: this
+ * is an interface choice of the library, not a step of the method.
+ *   Arguments and outputs are those of vp_router, minus ws / ws_bytes; the results are the
+ *   same.  The router's scratch comes from one fixed device buffer inside the library,
+ *   large enough for up to 32 heads (about 1.56 MiB, held on every GPU that loads the
+ *   library until the process exits); a call that would need more returns
+ *   VP_ERR_STATIC_SCRATCH.  The call allocates nothing (no cudaMalloc, cudaFree or
+ *   allocating library routine).
+ *   The first call on a device looks up the buffer's device address (set-up, once per
+ *   device, with that device current); make that first call before any stream capture.
+ *   All calls on a device share the buffer, which keeps the last call's contents; the parts
+ *   that must start at zero are cleared at the start of every call.  Calls that overlap on
+ *   the GPU (unordered streams or host threads) race on the buffer: serialise them.
+ *   Device error bits (e.g. a NaN saliency) are cleared per call and not reported.
+ */
+vp_status vp_router_noalloc(const vp_dims* dims, const vp_bf16* qkv, const vp_router_weights* rw,
+                            const int32_t* force_modes, float* s, int32_t* modes, float* q_pool,
+                            float* ctx, float* mean_v, float* r, void* stream);
 
 /* Kernel classes reported by the launch profiler. */
 #define VP_KERNEL_GEMM 0

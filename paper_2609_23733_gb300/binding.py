@@ -25,7 +25,7 @@ KERNEL_CLASSES = ["gemm", "router_pool", "router_keys", "router_r", "bin_heads",
 
 STATUS = {0: "VP_OK", 1: "VP_ERR_INVALID_ARG", 2: "VP_ERR_UNSUPPORTED_SHAPE", 3: "VP_ERR_ALIGNMENT",
           4: "VP_ERR_CUDA", 5: "VP_ERR_DEVICE_TIMEOUT", 6: "VP_ERR_WORKSPACE",
-          7: "VP_ERR_UNSUPPORTED_DEVICE"}
+          7: "VP_ERR_UNSUPPORTED_DEVICE", 8: "VP_ERR_STATIC_SCRATCH"}
 
 
 class VPError(RuntimeError):
@@ -63,6 +63,9 @@ _SIGS = [
     ("vp_router", c_int32, [POINTER(VpDims), c_void_p, POINTER(VpRouterWeights), c_void_p, c_void_p,
                             c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
                             c_void_p]),
+    ("vp_router_noalloc", c_int32, [POINTER(VpDims), c_void_p, POINTER(VpRouterWeights), c_void_p,
+                                    c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                    c_void_p]),
     ("vp_bin_heads", c_int32, [c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                c_void_p]),
     ("vp_head_attention", c_int32, [POINTER(VpDims), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
@@ -189,6 +192,15 @@ def vp_router(dm, qkv, rw: VpRouterWeights, force_modes, s, modes, q_pool, ctx, 
     _check(lib().vp_router(ctypes.byref(dm), _p(qkv), ctypes.byref(rw), _p(force_modes), _p(s), _p(modes),
                            _p(q_pool), _p(ctx), _p(mean_v), _p(r), _p(ws), ws.numel(), _stream(stream)),
            "vp_router")
+
+
+def vp_router_noalloc(dm, qkv, rw: VpRouterWeights, force_modes, s, modes, q_pool, ctx, mean_v, r,
+                      stream=None):
+    """vp_router without a workspace: scratch comes from a fixed buffer inside the library,
+    for callers that cannot allocate device memory (see include/vp.h)."""
+    _check(lib().vp_router_noalloc(ctypes.byref(dm), _p(qkv), ctypes.byref(rw), _p(force_modes), _p(s),
+                                   _p(modes), _p(q_pool), _p(ctx), _p(mean_v), _p(r), _stream(stream)),
+           "vp_router_noalloc")
 
 
 def vp_bin_heads(H, N, modes, head_ids, offsets, work=None, n_work=None, stream=None):

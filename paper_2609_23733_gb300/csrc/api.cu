@@ -285,6 +285,7 @@ const char* vp_status_string(vp_status s) {
     case VP_ERR_DEVICE_TIMEOUT: return "device wait timed out";
     case VP_ERR_WORKSPACE: return "workspace missing or too small";
     case VP_ERR_UNSUPPORTED_DEVICE: return "device is not sm_103";
+    case VP_ERR_STATIC_SCRATCH: return "needs more scratch than the fixed no-allocation buffer holds";
   }
   return "unknown status";
 }
