@@ -1,21 +1,25 @@
 // Full-mode heads (Algorithm 1, step 2, s_h >= tau_high): Y_h = softmax(Q_h K_h^T / sqrt d) V_h
 // as a flash-attention kernel on the sm_103a tensor cores.
 //
-// Persistent CTAs (one per SM) walk the work list of (full head, 128-query tile) pairs
-// read from the device bins.  Warp roles:
-//   warp 0     TMA producer: Q tile once per item, K/V tiles through a 3-stage ring.
-//   warp 1     owns TMEM; one lane issues tcgen05.mma: S = Q K^T into one of two TMEM
-//              S buffers (128 x 128 fp32 each), O += P V into a TMEM O buffer (128 x 64).
-//   warps 2-5  softmax: each thread owns one query row (its TMEM lane), reads its S row,
-//              keeps the running max / sum (online softmax, max rescaled lazily: O and the
-//              sum are rescaled only when the max grows by more than 2^8), writes P as
-//              bf16 into one of two 128-byte-swizzled smem buffers, and at the end
-//              normalises O and stores Y rows.
-// The S MMA of tile j+1 is issued before the P V MMA of tile j, so the tensor core works
-// on the next scores while the softmax warps process the current ones.  Keys past N are
-// zero-filled by TMA and masked to -inf; query rows past N are not stored.
-// Every mbarrier wait is bounded (see mbar_wait); on timeout the CTA records the error,
-// stops issuing work, waits for its own outstanding copies and MMAs, frees TMEM and exits.
+// Persistent CTAs (one per SM) walk the work items (full head, pair of 128-query tiles)
+// read from the device bins.  The two query tiles of an item run as two independent
+// chains, c = 0 and c = 1, that share the K/V pipeline:
+//   warp 0        TMA producer: both Q tiles once per item, K/V tiles through a 4-stage ring.
+//   warp 1        TMEM owner.  Warps 1 and 2: one lane each issues chain c's tcgen05.mma:
+//                 S_c = Q_c K^T (SS form, 128 x 128 fp32 in TMEM) and O_c += P_c V
+//                 (TS form: P_c read from TMEM as bf16, V from shared memory, MN-major).
+//   warps 4-7     softmax of chain 0, warps 8-11 softmax of chain 1: one query row per
+//                 thread (its TMEM lane).  The thread loads its S row, takes the max (3-input
+//                 max), computes 2^(s c - m) (packed f32x2 FMA + MUFU ex2), sums with packed
+//                 adds, and writes P as bf16 pairs back to TMEM.  The running max is
+//                 rescaled lazily: O and the sum are rescaled only when the max grows by
+//                 more than 2^8; otherwise the stale max is kept (exact either way).
+// While one chain's softmax runs, the tensor core works on the other chain's S and P V
+// products, and S_c(j+1) is issued as soon as chain c has read S_c(j).
+// TMEM: S_0 [0,128) S_1 [128,256) O_0 [256,320) O_1 [320,384) P_0 [384,448) P_1 [448,512).
+// Keys past N are zero-filled by TMA and masked to -inf; query rows past N are not stored.
+// Every mbarrier wait is bounded (mbar_wait); on timeout the CTA records the error, stops
+// issuing work, waits (bounded) for its own outstanding copies and MMAs, frees TMEM, exits.
 #include <math.h>
 
 #include "common.cuh"
@@ -25,23 +29,22 @@ namespace vp {
 
 namespace {
 
-constexpr int kBM = 128;      // query rows per tile
-constexpr int kBN = 128;      // keys per tile
-constexpr int kStages = 3;    // K/V ring depth
-constexpr int kTileBytes = 128 * 64 * 2;   // one 128 x 64 bf16 tile (16 KB)
+constexpr int kBM = 128;       // query rows per tile (two tiles per item)
+constexpr int kBN = 128;       // keys per tile
+constexpr int kStages = 4;     // K/V ring depth
+constexpr int kTileBytes = 128 * 64 * 2;  // one 128 x 64 bf16 tile (16 KB)
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTmemO = 256;          // O accumulator column offset
+constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr float kRescaleThreshold = 8.f;  // log2 units
+constexpr int kThreads = 384;
 
 struct FullSmem {
-  __nv_bfloat16 q[128 * 64];
+  __nv_bfloat16 q[2][128 * 64];
   __nv_bfloat16 k[kStages][128 * 64];
   __nv_bfloat16 v[kStages][128 * 64];
-  __nv_bfloat16 p[2][2][128 * 64];  // [buffer][key half] 128 rows x 64 keys, swizzled
   uint64_t q_full, q_empty;
   uint64_t k_full[kStages], v_full[kStages], kv_empty[kStages];
-  uint64_t s_full[2], s_empty[2], p_full[2], o_bar[2];
-  uint64_t o_empty, drain;
+  uint64_t s_full[2], s_empty[2], p_full[2], o_bar[2], o_empty[2], drain[2];
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -54,7 +57,13 @@ struct FullParams {
   unsigned int* err;
 };
 
-__global__ void __launch_bounds__(192, 1)
+__device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity, unsigned int* err,
+                                         volatile int* abort_flag) {
+  const bool ok = mbar_wait(bar, parity, err, abort_flag);
+  return __all_sync(0xffffffffu, ok);  // TMEM access below is warp-collective
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
     attn_full_kernel(const __grid_constant__ CUtensorMap tmap_qkv, FullParams prm) {
   extern __shared__ unsigned char smem_raw[];
   FullSmem& sm = *reinterpret_cast<FullSmem*>(
@@ -63,9 +72,9 @@ __global__ void __launch_bounds__(192, 1)
   const int first = __ldg(prm.offsets + 2);
   const int n_heads = __ldg(prm.offsets + 3) - first;
   const int N = prm.N, H = prm.H;
-  const int n_qt = (N + kBM - 1) / kBM;
+  const int n_pairs = (N + 2 * kBM - 1) / (2 * kBM);
   const int n_kv = (N + kBN - 1) / kBN;
-  const int items = n_heads * n_qt;
+  const int items = n_heads * n_pairs;
   if ((int)blockIdx.x >= items) return;  // uniform across the CTA
 
   const int warp = warp_id(), lane = lane_id();
@@ -73,20 +82,20 @@ __global__ void __launch_bounds__(192, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
-    mbar_init(&sm.q_empty, 1);
+    mbar_init(&sm.q_empty, 2);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+      mbar_init(&sm.kv_empty[s], 2);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&sm.s_full[b], 1);
-      mbar_init(&sm.s_empty[b], 128);
-      mbar_init(&sm.p_full[b], 128);
-      mbar_init(&sm.o_bar[b], 1);
+    for (int c = 0; c < 2; ++c) {
+      mbar_init(&sm.s_full[c], 1);
+      mbar_init(&sm.s_empty[c], 128);
+      mbar_init(&sm.p_full[c], 128);
+      mbar_init(&sm.o_bar[c], 1);
+      mbar_init(&sm.o_empty[c], 128);
+      mbar_init(&sm.drain[c], 1);
     }
-    mbar_init(&sm.o_empty, 128);
-    mbar_init(&sm.drain, 1);
     sm.abort_flag = 0;
     fence_mbarrier_init();
     fence_proxy_async_smem();
@@ -104,20 +113,19 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      uint32_t lc = 0, ic = 0, q_issued = 0;
+      uint32_t lc = 0, ic = 0;
       bool ok = true;
       for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
-        const int h = __ldg(prm.head_ids + first + item / n_qt);
-        const int qt = item % n_qt;
+        const int h = __ldg(prm.head_ids + first + item / n_pairs);
+        const int qp = item % n_pairs;
         ok = mbar_wait(&sm.q_empty, (ic & 1) ^ 1, prm.err, abort_flag);
         if (!ok) break;
-        ++q_issued;
-        mbar_arrive_expect_tx(&sm.q_full, kTileBytes);
-        tma_load_2d(sm.q, &tmap_qkv, &sm.q_full, h * 64, qt * kBM);
+        mbar_arrive_expect_tx(&sm.q_full, 2 * kTileBytes);
+        tma_load_2d(sm.q[0], &tmap_qkv, &sm.q_full, h * 64, qp * 2 * kBM);
+        tma_load_2d(sm.q[1], &tmap_qkv, &sm.q_full, h * 64, qp * 2 * kBM + kBM);
         for (int j = 0; j < n_kv; ++j, ++lc) {
           const int st = lc % kStages;
-          const uint32_t rnd = lc / kStages;
-          ok = mbar_wait(&sm.kv_empty[st], (rnd & 1) ^ 1, prm.err, abort_flag);
+          ok = mbar_wait(&sm.kv_empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
           if (!ok) break;
           mbar_arrive_expect_tx(&sm.k_full[st], kTileBytes);
           tma_load_2d(sm.k[st], &tmap_qkv, &sm.k_full[st], (H + h) * 64, j * kBN);
@@ -127,8 +135,11 @@ __global__ void __launch_bounds__(192, 1)
       }
       if (!ok) {
         // Let the copies this thread issued land before the CTA releases its smem.
-        if (q_issued > 0)
-          for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.q_full, (q_issued - 1) & 1); ++t) {}
+        // ic counts items whose Q load was issued when the loop broke inside the K/V loop,
+        // and items + 1 when it broke at the Q wait; waiting on the last issued phase is
+        // bounded either way.
+        if (ic > 0)
+          for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.q_full, (ic - 1) & 1); ++t) {}
         for (int s = 0; s < kStages; ++s) {
           if (lc > (uint32_t)s) {
             const uint32_t last = (lc - 1 - s) / kStages * kStages + s;  // last use of stage s
@@ -139,179 +150,177 @@ __global__ void __launch_bounds__(192, 1)
         }
       }
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 || warp == 2) {
+    // ------------------------------------------------------------ MMA issuers (chain c)
+    const int c = warp - 1;
     if (lane == 0) {
-      const uint32_t id_s = idesc_bf16(kBM, kBN, 0, 0);   // Q (K-major) x K^T (K-major)
-      const uint32_t id_o = idesc_bf16(kBM, 64, 0, 1);    // P (K-major) x V (MN-major)
-      const uint64_t dq = sdesc_sw128(smem_u32(sm.q));
-      uint32_t lc = 0, ic = 0, g = 0;  // g: global tile counter (S / P / O buffers)
+      const uint32_t id_s = idesc_bf16(kBM, kBN, 0, 0);  // Q (K-major) x K^T (K-major)
+      const uint32_t id_o = idesc_bf16(kBM, 64, 0, 1);   // P (TMEM) x V (MN-major)
+      const uint64_t dq = sdesc_sw128(smem_u32(sm.q[c]));
+      const uint32_t t_s = tmem + kColS + c * kBN;
+      const uint32_t t_o = tmem + kColO + c * 64;
+      const uint32_t t_p = tmem + kColP + c * 64;
+      uint32_t lc = 0, ic = 0, g = 0;  // K/V tiles seen, items, S/P/O tiles of this chain
       bool ok = true;
       for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
         ok = mbar_wait(&sm.q_full, ic & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
         const uint32_t lc0 = lc, g0 = g;
-        // S_j = Q K_j^T into S buffer (g0 + j) & 1.
         auto issue_s = [&](int j) -> bool {
           const uint32_t l = lc0 + j, gg = g0 + j;
           const int st = l % kStages;
           if (!mbar_wait(&sm.k_full[st], (l / kStages) & 1, prm.err, abort_flag)) return false;
-          if (!mbar_wait(&sm.s_empty[gg & 1], ((gg >> 1) & 1) ^ 1, prm.err, abort_flag)) return false;
+          if (!mbar_wait(&sm.s_empty[c], (gg & 1) ^ 1, prm.err, abort_flag)) return false;
           tc_fence_after();
           const uint64_t dk = sdesc_sw128(smem_u32(sm.k[st]));
-          const uint32_t d_s = tmem + (gg & 1) * kBN;
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)  // 4 x K=16 covers d = 64; +32 bytes per step
-            tc_mma_ss(d_s, dq + 2 * kk, dk + 2 * kk, id_s, kk > 0);
-          tc_commit(&sm.s_full[gg & 1]);
+          for (int kk = 0; kk < 4; ++kk)  // 4 x K=16 covers d = 64 (+32 bytes per step)
+            tc_mma_ss(t_s, dq + 2 * kk, dk + 2 * kk, id_s, kk > 0);
+          tc_commit(&sm.s_full[c]);
           if (j == n_kv - 1) tc_commit(&sm.q_empty);
           return true;
         };
         ok = issue_s(0);
         for (int j = 0; j < n_kv && ok; ++j) {
           if (j + 1 < n_kv) {
-            ok = issue_s(j + 1);
+            ok = issue_s(j + 1);  // as soon as the softmax has read S_c(j)
             if (!ok) break;
           }
-          // O (+)= P_j V_j
           const uint32_t l = lc0 + j, gg = g0 + j;
           const int st = l % kStages;
-          ok = mbar_wait(&sm.p_full[gg & 1], (gg >> 1) & 1, prm.err, abort_flag) &&
+          ok = mbar_wait(&sm.p_full[c], gg & 1, prm.err, abort_flag) &&
                mbar_wait(&sm.v_full[st], (l / kStages) & 1, prm.err, abort_flag) &&
-               (j > 0 || mbar_wait(&sm.o_empty, (ic & 1) ^ 1, prm.err, abort_flag));
+               (j > 0 || mbar_wait(&sm.o_empty[c], (ic & 1) ^ 1, prm.err, abort_flag));
           if (!ok) break;
           tc_fence_after();
-          const uint32_t pb0 = smem_u32(sm.p[gg & 1][0]);
           const uint64_t dv = sdesc_sw128(smem_u32(sm.v[st]));
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {  // 8 x K=16 covers 128 keys
-            const uint64_t da = sdesc_sw128(pb0 + (kk >> 2) * kTileBytes) + 2 * (kk & 3);
-            const uint64_t db = dv + (uint64_t)(kk * 16 * 128 / 16);  // 16 keys = 2048 bytes
-            tc_mma_ss(tmem + kTmemO, da, db, id_o, (j > 0 || kk > 0) ? 1u : 0u);
-          }
-          tc_commit(&sm.o_bar[gg & 1]);
+          for (int kk = 0; kk < 8; ++kk)  // 8 x K=16 covers 128 keys: 8 TMEM columns, 2 KB of V
+            tc_mma_ts(t_o, t_p + 8 * kk, dv + (uint64_t)(kk * 128), id_o,
+                      (j > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(&sm.o_bar[c]);
           tc_commit(&sm.kv_empty[st]);
         }
         lc = lc0 + n_kv;
         g = g0 + n_kv;
       }
       if (!ok) {
-        // Wait (bounded) for every MMA this thread issued before TMEM is released.
-        tc_commit(&sm.drain);
-        for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.drain, 0); ++t) {}
+        tc_commit(&sm.drain[c]);
+        for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.drain[c], 0); ++t) {}
       }
     }
-  } else {
+  } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax / epilogue
-    const int quarter = warp & 3;  // TMEM lane quarter this warp may access
+    const int c = (warp - 4) >> 2;  // chain
+    const int quarter = warp & 3;   // TMEM lane quarter this warp may access
     const int row_in_tile = quarter * 32 + lane;
-    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
-    const float c = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
-    const int n_tail = N - (n_kv - 1) * kBN;       // valid keys in the last tile
-    uint32_t g = 0, ic = 0;
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    const uint32_t t_s = tmem + lane_off + kColS + c * kBN;
+    const uint32_t t_o = tmem + lane_off + kColO + c * 64;
+    const uint32_t t_p = tmem + lane_off + kColP + c * 64;
+    const float cs = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
+    const int n_tail = N - (n_kv - 1) * kBN;        // valid keys in the last tile
+    uint32_t g = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
-      const int h = __ldg(prm.head_ids + first + item / n_qt);
-      const int qt = item % n_qt;
+    for (int item = blockIdx.x; item < items && ok; item += gridDim.x) {
+      const int h = __ldg(prm.head_ids + first + item / n_pairs);
+      const int qp = item % n_pairs;
       float m = 0.f, lsum = 0.f;
       for (int j = 0; j < n_kv; ++j, ++g) {
-        const int b = g & 1;
-        ok = mbar_wait(&sm.s_full[b], (g >> 1) & 1, prm.err, abort_flag);
-        ok = __all_sync(0xffffffffu, ok);  // TMEM loads below need the whole warp
+        ok = wait_all(&sm.s_full[c], g & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
         float s[128];
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) tmem_ld32(t_lane + b * kBN + 32 * cc, s + 32 * cc);
+        for (int cc = 0; cc < 4; ++cc) tmem_ld32(t_s + 32 * cc, s + 32 * cc);
         tmem_wait_ld();
         tc_fence_before();
-        mbar_arrive(&sm.s_empty[b]);
+        mbar_arrive(&sm.s_empty[c]);  // the MMA warp may overwrite S_c now
         if (j == n_kv - 1 && n_tail < kBN) {
 #pragma unroll
           for (int i = 0; i < 128; ++i)
             if (i >= n_tail) s[i] = -INFINITY;
         }
-        float mx = s[0];
+        // Row max: eight independent 3-input max chains, then a short tree.
+        float mx;
+        {
+          float t[8];
 #pragma unroll
-        for (int i = 1; i < 128; ++i) mx = fmaxf(mx, s[i]);
-        const float mx2 = mx * c;
+          for (int k = 0; k < 8; ++k) t[k] = s[k];
+#pragma unroll
+          for (int i = 8; i < 128; i += 16) {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) t[k] = fmax3(t[k], s[i + k], s[i + 8 + k]);
+          }
+          mx = fmaxf(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], fmax3(t[5], t[6], t[7])));
+        }
+        const float mx2 = mx * cs;
+        float alpha = 1.f;
+        bool need = false;
         if (j == 0) {
           m = mx2;
-        } else {
-          const bool need = mx2 > m + kRescaleThreshold;
-          if (__any_sync(0xffffffffu, need)) {
-            // Rescale O (and the sum) after P_{j-1} V_{j-1} has landed in TMEM.
-            const uint32_t gp = g - 1;
-            ok = mbar_wait(&sm.o_bar[gp & 1], (gp >> 1) & 1, prm.err, abort_flag);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) break;
-            tc_fence_after();
-            const float alpha = need ? fast_exp2(m - mx2) : 1.f;
-            float o[64];
-            tmem_ld32(t_lane + kTmemO, o);
-            tmem_ld32(t_lane + kTmemO + 32, o + 32);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 64; ++i) o[i] *= alpha;
-            tmem_st32(t_lane + kTmemO, o);
-            tmem_st32(t_lane + kTmemO + 32, o + 32);
-            tmem_wait_st();
-            if (need) {
-              lsum *= alpha;
-              m = mx2;
-            }
-          }
+        } else if (mx2 > m + kRescaleThreshold) {
+          need = true;
+          alpha = fast_exp2(m - mx2);
+          m = mx2;
         }
-        float part = 0.f;
+        // p = 2^(s cs - m), summed in packed pairs.
+        const float2 c2 = make_float2(cs, cs), nm = make_float2(-m, -m);
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int i = 0; i < 128; ++i) {
-          s[i] = fast_exp2(fmaf(s[i], c, -m));
-          part += s[i];
+        for (int i = 0; i < 64; ++i) {
+          float2 x = ffma2(make_float2(s[2 * i], s[2 * i + 1]), c2, nm);
+          x.x = fast_exp2(x.x);
+          x.y = fast_exp2(x.y);
+          s[2 * i] = x.x;
+          s[2 * i + 1] = x.y;
+          if (i & 1)
+            acc1 = fadd2(acc1, x);
+          else
+            acc0 = fadd2(acc0, x);
         }
-        lsum += part;
-        // P buffer b is free once P_{g-2} V_{g-2} has completed.
-        if (g >= 2) {
-          ok = mbar_wait(&sm.o_bar[b], ((g - 2) >> 1) & 1, prm.err, abort_flag);
-          ok = __all_sync(0xffffffffu, ok);
+        const float2 at = fadd2(acc0, acc1);
+        lsum = lsum * alpha + (at.x + at.y);
+        // P_c and O_c are free once P_c(g-1) V has completed.
+        if (g > 0) {
+          ok = wait_all(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
           if (!ok) break;
+          tc_fence_after();
         }
-        {
-          unsigned char* pb = reinterpret_cast<unsigned char*>(sm.p[b][0]);
-          const int rsw = row_in_tile & 7;
-          const uint32_t row_off = (row_in_tile >> 3) * 1024 + rsw * 128;
 #pragma unroll
-          for (int half = 0; half < 2; ++half) {
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t pk[16];
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch) {
-              const float* src = s + 64 * half + 8 * ch;
-              uint4 v;
-              v.x = pack_bf16x2(src[0], src[1]);
-              v.y = pack_bf16x2(src[2], src[3]);
-              v.z = pack_bf16x2(src[4], src[5]);
-              v.w = pack_bf16x2(src[6], src[7]);
-              *reinterpret_cast<uint4*>(pb + half * kTileBytes + row_off + ((ch ^ rsw) << 4)) = v;
-            }
-          }
+          for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(s[32 * cc + 2 * i], s[32 * cc + 2 * i + 1]);
+          tmem_st16(t_p + 16 * cc, pk);
         }
-        fence_proxy_async_smem();
+        if (__any_sync(0xffffffffu, need)) {
+          float o[64];
+          tmem_ld32(t_o, o);
+          tmem_ld32(t_o + 32, o + 32);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 64; ++i) o[i] *= alpha;
+          tmem_st32(t_o, o);
+          tmem_st32(t_o + 32, o + 32);
+        }
+        tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(&sm.p_full[b]);
+        mbar_arrive(&sm.p_full[c]);
       }
       if (!ok) break;
       // Epilogue: O / sum -> bf16 -> Y[row][h][:]
-      const uint32_t gl = g - 1;
-      ok = mbar_wait(&sm.o_bar[gl & 1], (gl >> 1) & 1, prm.err, abort_flag);
-      ok = __all_sync(0xffffffffu, ok);
+      ok = wait_all(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
       float o[64];
-      tmem_ld32(t_lane + kTmemO, o);
-      tmem_ld32(t_lane + kTmemO + 32, o + 32);
+      tmem_ld32(t_o, o);
+      tmem_ld32(t_o + 32, o + 32);
       tmem_wait_ld();
       tc_fence_before();
-      mbar_arrive(&sm.o_empty);
-      const int row = qt * kBM + row_in_tile;
+      mbar_arrive(&sm.o_empty[c]);
+      const int row = qp * 2 * kBM + c * kBM + row_in_tile;
       if (row < N) {
         const float inv = 1.f / lsum;
         uint4* dst = reinterpret_cast<uint4*>(prm.y + ((size_t)row * H + h) * 64);
@@ -325,6 +334,7 @@ __global__ void __launch_bounds__(192, 1)
           dst[ch] = v;
         }
       }
+      __syncwarp();
     }
   }
 
@@ -348,7 +358,7 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
   if (e != cudaSuccess) return e;
   FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.err};
   prof_before(VP_KERNEL_ATTN_FULL, st);
-  attn_full_kernel<<<num_sms, 192, smem, st>>>(tmap, prm);
+  attn_full_kernel<<<num_sms, kThreads, smem, st>>>(tmap, prm);
   prof_after(st);
   return cudaGetLastError();
 }
