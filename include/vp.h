@@ -178,7 +178,8 @@ vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32
  * Algorithm 1 (QKV, W_O, FFN) on tcgen05 tensor cores with fp32 accumulation.
  *   A [M][K] bf16, W [Nout][K] bf16 (nn.Linear layout), bias [Nout] float or NULL,
  *   act VP_ACT_NONE / VP_ACT_GELU, scale [Nout] float or NULL (1), residual [M][Nout]
- *   bf16 or NULL (0; may alias out), out [M][Nout] bf16.  K % 8 == 0, Nout % 8 == 0.
+ *   bf16 or NULL (0; may alias out), out [M][Nout] bf16.  K % 8 == 0, Nout % 8 == 0; every
+ *   pointer 16-byte aligned (the epilogue reads bias and scale four floats at a time).
  */
 vp_status vp_linear(int32_t M, int32_t Nout, int32_t K, const vp_bf16* A, const vp_bf16* W,
                     const float* bias, int32_t act, const float* scale, const vp_bf16* residual,

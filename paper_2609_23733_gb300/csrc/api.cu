@@ -90,7 +90,8 @@ int device_sm_count() { return dev_info().sms; }
 bool device_is_sm103() { return dev_info().sm103 == 1; }
 
 cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
-                              uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows) {
+                              uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows,
+                              int swizzle_bytes) {
   std::call_once(g_encode_once, [] {
     void* fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -106,7 +107,10 @@ cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols,
   const cuuint32_t estr[2] = {1, 1};
   CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
                         strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        swizzle_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                        : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                              : CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
@@ -413,7 +417,8 @@ vp_status vp_linear(int32_t M, int32_t Nout, int32_t K, const vp_bf16* A, const 
   if (M < 1 || Nout < 8 || K < 8 || Nout % 8 || K % 8) return VP_ERR_UNSUPPORTED_SHAPE;
   if (!A || !W || !out) return VP_ERR_INVALID_ARG;
   if (act != VP_ACT_NONE && act != VP_ACT_GELU) return VP_ERR_INVALID_ARG;
-  if (!aligned16(A) || !aligned16(W) || !aligned16(out) || (residual && !aligned16(residual)))
+  if (!aligned16(A) || !aligned16(W) || !aligned16(out) || (residual && !aligned16(residual)) ||
+      (bias && !aligned16(bias)) || (scale && !aligned16(scale)))
     return VP_ERR_ALIGNMENT;
   VP_TRY(check_device());
   unsigned int* err = nullptr;
@@ -454,7 +459,8 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
   VP_TRY(check_dims(dims));
   if (!x || !w_qkv || !w_o || !out) return VP_ERR_INVALID_ARG;
   if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(w_o) || !aligned16(out) ||
-      (qkv_out && !aligned16(qkv_out)) || (y_out && !aligned16(y_out)))
+      (qkv_out && !aligned16(qkv_out)) || (y_out && !aligned16(y_out)) ||
+      (b_qkv && !aligned16(b_qkv)) || (b_o && !aligned16(b_o)))
     return VP_ERR_ALIGNMENT;
   VP_TRY(check_router_weights(rw));
   VP_TRY(check_surrogate_weights(sw));
@@ -488,7 +494,10 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     if (!w.ln1_g || !w.ln1_b || !w.w_qkv || !w.w_o || !w.ls1 || !w.ln2_g || !w.ln2_b ||
         !w.w_fc1 || !w.w_fc2 || !w.ls2)
       return VP_ERR_INVALID_ARG;
-    if (!aligned16(w.w_qkv) || !aligned16(w.w_o) || !aligned16(w.w_fc1) || !aligned16(w.w_fc2))
+    if (!aligned16(w.w_qkv) || !aligned16(w.w_o) || !aligned16(w.w_fc1) || !aligned16(w.w_fc2) ||
+        !aligned16(w.ls1) || !aligned16(w.ls2) || (w.b_qkv && !aligned16(w.b_qkv)) ||
+        (w.b_o && !aligned16(w.b_o)) || (w.b_fc1 && !aligned16(w.b_fc1)) ||
+        (w.b_fc2 && !aligned16(w.b_fc2)))
       return VP_ERR_ALIGNMENT;
     VP_TRY(check_router_weights(&w.router));
     VP_TRY(check_surrogate_weights(&w.surrogate));

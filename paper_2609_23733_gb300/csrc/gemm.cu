@@ -3,8 +3,11 @@
 // Persistent CTAs (one per SM), 128 x 256 output tiles, 64-wide K blocks through a 4-stage
 // TMA ring (128-byte swizzle), tcgen05.mma (M=128, N=256, K=16, bf16 -> fp32) into one of
 // two TMEM accumulators, so the epilogue of tile i overlaps the main loop of tile i+1.
-// Warp roles: warp 0 TMA, warp 1 TMEM owner + MMA issue, warps 2-5 epilogue (one row per
-// thread: TMEM lane -> registers -> bias / GELU / LayerScale / residual -> bf16 stores).
+// Warp roles: warp 0 TMA, warp 1 TMEM owner + MMA issue, warps 2-9 epilogue: each owns a
+// (32-row TMEM lane quarter, 128-column half) of the tile, one row per thread; per 32-column
+// chunk it loads TMEM (the next chunk's load in flight while this one is processed), applies
+// bias / GELU / LayerScale / residual, packs bf16 into a 64-byte-swizzled 32 x 32 staging
+// block in shared memory and writes it with a TMA tensor store (clipped at the tensor edge).
 // Tiles are visited N-fastest so the CTAs in flight share A rows and all of W in L2.
 #include <math.h>
 
@@ -19,10 +22,13 @@ constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
 constexpr int kABytes = kBM * kBK * 2;  // 16 KB
 constexpr int kBBytes = kBN * kBK * 2;  // 32 KB
 constexpr uint32_t kTmemCols = 512;
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 
 struct GemmSmem {
   __nv_bfloat16 a[kStages][kBM * kBK];
   __nv_bfloat16 b[kStages][kBN * kBK];
+  __nv_bfloat16 stage[kEpiWarps][2][32 * 32];  // per epilogue warp: two 32 x 32 output blocks
   uint64_t full[kStages], empty[kStages];
   uint64_t acc_full[2], acc_empty[2], drain;
   uint32_t tmem_base;
@@ -43,9 +49,10 @@ __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
 }
 
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
-                const __grid_constant__ CUtensorMap tmap_b, GemmParams prm) {
+                const __grid_constant__ CUtensorMap tmap_b,
+                const __grid_constant__ CUtensorMap tmap_out, GemmParams prm) {
   extern __shared__ unsigned char smem_raw[];
   GemmSmem& sm = *reinterpret_cast<GemmSmem*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -64,7 +71,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&sm.acc_full[b], 1);
-      mbar_init(&sm.acc_empty[b], 128);
+      mbar_init(&sm.acc_empty[b], 32 * kEpiWarps);
     }
     mbar_init(&sm.drain, 1);
     sm.abort_flag = 0;
@@ -72,6 +79,7 @@ __global__ void __launch_bounds__(192, 1)
     fence_proxy_async_smem();
     tma_prefetch_desc(&tmap_a);
     tma_prefetch_desc(&tmap_b);
+    tma_prefetch_desc(&tmap_out);
   }
   if (warp == 1) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
@@ -138,9 +146,12 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else {
-    const int quarter = warp & 3;
+    const int e = warp - 2;                 // epilogue warp 0..7
+    const int quarter = warp & 3;           // TMEM lane quarter
+    const int half = e >> 2;                // column half of the tile
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
-    uint32_t i = 0;
+    unsigned char* stg = reinterpret_cast<unsigned char*>(&sm.stage[e][0][0]);
+    uint32_t i = 0, nst = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
       const int mt = t / n_tiles, nt = t - mt * n_tiles;
       const uint32_t ab = i & 1;
@@ -148,64 +159,93 @@ __global__ void __launch_bounds__(192, 1)
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
-      const int row = mt * kBM + quarter * 32 + lane;
+      const int row0 = mt * kBM + quarter * 32;
+      const int row = row0 + lane;
       const bool row_ok = row < M;
-      for (int cc = 0; cc < kBN / 32; ++cc) {
-        float v[32];
-        __syncwarp();  // TMEM loads are warp-collective; lanes may have skipped a chunk
-        tmem_ld32(t_lane + ab * kBN + cc * 32, v);
-        tmem_wait_ld();
-        if (cc == kBN / 32 - 1) {
-          tc_fence_before();
-          mbar_arrive(&sm.acc_empty[ab]);
-        }
-        const int col0 = nt * kBN + cc * 32;
-        if (!row_ok || col0 >= N) continue;
-        float res[32];
-        const bool full_chunk = col0 + 32 <= N;
-        if (prm.residual) {
-          const __nv_bfloat16* rp = prm.residual + (size_t)row * N + col0;
-          if (full_chunk) {
+      const uint32_t tcol = t_lane + ab * kBN + half * 128;
+      float v[2][32];
+      tmem_ld32(tcol, v[0]);
+      tmem_wait_ld();
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        if (cc + 1 < 4) tmem_ld32(tcol + 32 * (cc + 1), v[(cc + 1) & 1]);  // in flight meanwhile
+        float* x = v[cc & 1];
+        const int col0 = nt * kBN + half * 128 + cc * 32;
+        if (col0 < N) {
+          if (prm.bias) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const float4 b4 = col0 + 4 * q + 3 < N
+                                    ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
+                                    : make_float4(0.f, 0.f, 0.f, 0.f);
+              x[4 * q] += b4.x;
+              x[4 * q + 1] += b4.y;
+              x[4 * q + 2] += b4.z;
+              x[4 * q + 3] += b4.w;
+            }
+          }
+          if (prm.act == VP_ACT_GELU) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) x[k] = gelu_erf(x[k]);
+          }
+          if (prm.scale) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const float4 s4 = col0 + 4 * q + 3 < N
+                                    ? __ldg(reinterpret_cast<const float4*>(prm.scale + col0) + q)
+                                    : make_float4(0.f, 0.f, 0.f, 0.f);
+              x[4 * q] *= s4.x;
+              x[4 * q + 1] *= s4.y;
+              x[4 * q + 2] *= s4.z;
+              x[4 * q + 3] *= s4.w;
+            }
+          }
+          if (prm.residual && row_ok) {
+            const __nv_bfloat16* rp = prm.residual + (size_t)row * N + col0;
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-              const uint4 u = *reinterpret_cast<const uint4*>(rp + 8 * q);
-              const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
+              if (col0 + 8 * q + 7 < N) {
+                const uint4 u = *reinterpret_cast<const uint4*>(rp + 8 * q);
+                const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                res[8 * q + 2 * e] = bf16_lo(uw[e]);
-                res[8 * q + 2 * e + 1] = bf16_hi(uw[e]);
+                for (int k = 0; k < 4; ++k) {
+                  x[8 * q + 2 * k] += bf16_lo(uw[k]);
+                  x[8 * q + 2 * k + 1] += bf16_hi(uw[k]);
+                }
               }
             }
-          } else {
-            for (int e = 0; e < 32; ++e) res[e] = col0 + e < N ? __bfloat162float(rp[e]) : 0.f;
           }
-        }
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int col = min(col0 + e, N - 1);
-          float x = v[e];
-          if (prm.bias) x += __ldg(prm.bias + col);
-          if (prm.act == VP_ACT_GELU) x = gelu_erf(x);
-          if (prm.scale) x *= __ldg(prm.scale + col);
-          if (prm.residual) x += res[e];
-          v[e] = x;
-        }
-        __nv_bfloat16* op = prm.out + (size_t)row * N + col0;
-        if (full_chunk) {
+          // Stage the 32 x 32 block (row = lane, 64 bytes) in the 64-byte swizzle the
+          // output tensor map uses: 16-byte chunk q of row r sits at chunk q ^ ((r >> 1) & 3).
+          unsigned char* buf = stg + (nst & 1) * 2048;
+          if (lane == 0 && nst >= 2) tma_store_wait_read<1>();  // this buffer's last store read it
+          __syncwarp();
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             uint4 u;
-            u.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
-            u.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
-            u.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
-            u.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
-            *reinterpret_cast<uint4*>(op + 8 * q) = u;
+            u.x = pack_bf16x2(x[8 * q + 0], x[8 * q + 1]);
+            u.y = pack_bf16x2(x[8 * q + 2], x[8 * q + 3]);
+            u.z = pack_bf16x2(x[8 * q + 4], x[8 * q + 5]);
+            u.w = pack_bf16x2(x[8 * q + 6], x[8 * q + 7]);
+            *reinterpret_cast<uint4*>(buf + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = u;
           }
-        } else {
-          for (int e = 0; e < 32 && col0 + e < N; ++e) op[e] = __float2bfloat16_rn(v[e]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmap_out, buf, col0, row0);
+            tma_store_commit();
+          }
+          ++nst;
+        }
+        tmem_wait_ld();
+        if (cc == 3) {
+          tc_fence_before();
+          mbar_arrive(&sm.acc_empty[ab]);
         }
       }
     }
+    if (lane == 0) tma_store_wait_all();
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -219,10 +259,12 @@ __global__ void __launch_bounds__(192, 1)
 }  // namespace
 
 cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, to;
   cudaError_t e = make_tmap_bf16_2d(&ta, a.A, (uint64_t)a.K, (uint64_t)a.M, (uint64_t)a.K, kBK, kBM);
   if (e != cudaSuccess) return e;
   e = make_tmap_bf16_2d(&tb, a.W, (uint64_t)a.K, (uint64_t)a.N, (uint64_t)a.K, kBK, kBN);
+  if (e != cudaSuccess) return e;
+  e = make_tmap_bf16_2d(&to, a.out, (uint64_t)a.N, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 64);
   if (e != cudaSuccess) return e;
   const int smem = (int)sizeof(GemmSmem) + 1024;
   e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -230,7 +272,7 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   const int tiles = ((a.M + kBM - 1) / kBM) * ((a.N + kBN - 1) / kBN);
   GemmParams prm{a.M, a.N, a.K, a.bias, a.act, a.scale, a.residual, a.out, a.err};
   prof_before(VP_KERNEL_GEMM, st);
-  gemm_kernel<<<min(num_sms, tiles), 192, smem, st>>>(ta, tb, prm);
+  gemm_kernel<<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
   prof_after(st);
   return cudaGetLastError();
 }

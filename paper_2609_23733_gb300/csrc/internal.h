@@ -107,7 +107,8 @@ cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float*
 // 2-D bf16 tensor [rows][cols] with a row pitch of `pitch_elems`, box of box_cols x box_rows,
 // 128-byte swizzle, zero fill out of bounds.
 cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols, uint64_t rows,
-                              uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows);
+                              uint64_t pitch_elems, uint32_t box_cols, uint32_t box_rows,
+                              int swizzle_bytes = 128);
 
 // Launch profiler hooks (no-ops unless vp_profile_begin is active).
 void prof_before(int kind, cudaStream_t st);
