@@ -383,7 +383,26 @@ def kernel_case(args):
     dev = torch.device("cuda:0")
     N = args.case_tokens
     qkv = torch.randn(N, 3 * D, device=dev).to(torch.bfloat16)
-    if args.kernel_case == "attn_full":
+    if args.kernel_case in ("layer_norm", "router", "surrogate"):
+        w = vpb.to_device(synth.make_layer_weights(synth.rng(0), block=True), dev)
+        dm = vpb.dims(N, H)
+        ws = vpb.workspace(dm, vpb.VP_WS_ROUTER, dev)
+        x = torch.randn(N, D, device=dev).to(torch.bfloat16)
+        y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+        s = torch.zeros(H, device=dev)
+        modes = torch.zeros(H, dtype=torch.int32, device=dev)
+        ctx = torch.zeros(H, d, device=dev)
+        mv = torch.zeros(H, d, device=dev)
+        ids = torch.arange(H, dtype=torch.int32, device=dev)
+        off = torch.tensor([0, 0, H, H], dtype=torch.int32, device=dev)
+        for _ in range(args.case_launches):
+            if args.kernel_case == "layer_norm":
+                vpb.vp_layer_norm(x, w["ln1_g"], w["ln1_b"], 1e-6, out=y)
+            elif args.kernel_case == "router":
+                vpb.vp_router(dm, qkv, vpb.router_weights(w), None, s, modes, None, ctx, mv, None, ws)
+            else:
+                vpb.vp_head_attention(dm, qkv, ids, off, ctx, mv, vpb.surrogate_weights(w), y, ws)
+    elif args.kernel_case == "attn_full":
         w = vpb.to_device(synth.make_layer_weights(synth.rng(0)), dev)
         y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
         dm = vpb.dims(N, H)
@@ -430,7 +449,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--full-layer", action="store_true", default=True)
     ap.add_argument("--no-full-layer", dest="full_layer", action="store_false")
-    ap.add_argument("--kernel-case", choices=["attn_full", "gemm"], default=None,
+    ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "layer_norm", "router", "surrogate"],
+                    default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
     ap.add_argument("--case-tokens", type=int, default=32768)
     ap.add_argument("--case-launches", type=int, default=2)

@@ -186,7 +186,8 @@ vp_status vp_linear(int32_t M, int32_t Nout, int32_t K, const vp_bf16* A, const 
                     vp_bf16* out, void* stream);
 
 /* vp_layer_norm -- out = LN(x) over rows of length D (biased variance, eps), bf16 in/out,
-   gamma / beta [D] float (Algorithm 1 steps 1 and 4).  D in {256, 512, 768, 1024, 2048, 4096}. */
+   gamma / beta [D] float (Algorithm 1 steps 1 and 4).  D in {256, 512, 768, 1024, 2048, 4096};
+   all pointers 16-byte aligned. */
 vp_status vp_layer_norm(int32_t M, int32_t D, const vp_bf16* x, const float* gamma,
                         const float* beta, float eps, vp_bf16* out, void* stream);
 
@@ -210,6 +211,7 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
  * [N][D] bf16.  layers: HOST array of n_layers vp_layer_weights (their tensors are device
  * pointers).  force_modes [n_layers][H] int32 or NULL; modes_out / s_out [n_layers][H] or
  * NULL.  ln_eps: LayerNorm epsilon (the paper does not state it; 1e-6 in the tests).
+ * Every weight, bias, LayerNorm and LayerScale pointer must be 16-byte aligned.
  */
 vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
                           const vp_layer_weights* layers, const int32_t* force_modes,

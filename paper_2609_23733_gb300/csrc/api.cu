@@ -443,7 +443,8 @@ vp_status vp_layer_norm(int32_t M, int32_t D, const vp_bf16* x, const float* gam
                         const float* beta, float eps, vp_bf16* out, void* stream) {
   if (M < 1 || !ln_width_supported(D)) return VP_ERR_UNSUPPORTED_SHAPE;
   if (!x || !gamma || !beta || !out) return VP_ERR_INVALID_ARG;
-  if (!aligned16(x) || !aligned16(out)) return VP_ERR_ALIGNMENT;
+  if (!aligned16(x) || !aligned16(out) || !aligned16(gamma) || !aligned16(beta))
+    return VP_ERR_ALIGNMENT;
   VP_TRY(check_device());
   return from_cuda(launch_layer_norm(M, D, reinterpret_cast<const __nv_bfloat16*>(x), gamma, beta,
                                      eps, reinterpret_cast<__nv_bfloat16*>(out),
@@ -495,7 +496,8 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
         !w.w_fc1 || !w.w_fc2 || !w.ls2)
       return VP_ERR_INVALID_ARG;
     if (!aligned16(w.w_qkv) || !aligned16(w.w_o) || !aligned16(w.w_fc1) || !aligned16(w.w_fc2) ||
-        !aligned16(w.ls1) || !aligned16(w.ls2) || (w.b_qkv && !aligned16(w.b_qkv)) ||
+        !aligned16(w.ls1) || !aligned16(w.ls2) || !aligned16(w.ln1_g) || !aligned16(w.ln1_b) ||
+        !aligned16(w.ln2_g) || !aligned16(w.ln2_b) || (w.b_qkv && !aligned16(w.b_qkv)) ||
         (w.b_o && !aligned16(w.b_o)) || (w.b_fc1 && !aligned16(w.b_fc1)) ||
         (w.b_fc2 && !aligned16(w.b_fc2)))
       return VP_ERR_ALIGNMENT;

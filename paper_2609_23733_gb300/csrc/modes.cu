@@ -68,14 +68,17 @@ struct SurrSmem {
   float ctx[64];
 };
 
-__global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
+constexpr int kSurrWarps = 8;
+constexpr int kSurrRows = 16 * kSurrWarps;  // rows per work item
+
+__global__ void __launch_bounds__(32 * kSurrWarps, 3) surrogate_heads_kernel(HeadAttnArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SurrSmem& sm = *reinterpret_cast<SurrSmem*>(smem_raw);
   const int first = __ldg(a.offsets + 1);
   const int n_heads = __ldg(a.offsets + 2) - first;
   const int N = a.N, H = a.H;
   const size_t row_pitch = (size_t)3 * H * kHeadDim;
-  const int chunks = (N + 63) / 64;
+  const int chunks = (N + kSurrRows - 1) / kSurrRows;
   const int items = n_heads * chunks;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int r = lane >> 2, c = lane & 3;
@@ -86,7 +89,7 @@ __global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
     const int h = __ldg(a.head_ids + first + slot);
     if (h != cur_h) {
       __syncthreads();  // previous head's weights no longer in use
-      for (int i = tid; i < 128 * 8; i += 128) {
+      for (int i = tid; i < 128 * 8; i += 32 * kSurrWarps) {
         const int row = i >> 3, ch = i & 7;
         const bool g = row < 64;
         const __nv_bfloat16* w1 = (g ? a.sw.g1_w : a.sw.d1_w) + ((size_t)h * 64 + (row & 63)) * 128 + ch * 8;
@@ -95,13 +98,13 @@ __global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
         *reinterpret_cast<uint4*>(&sm.w2[row * kBStride + ch * 8]) = __ldg(reinterpret_cast<const uint4*>(w2));
       }
       if (tid < 64) sm.ctx[tid] = __ldg(a.ctx + h * 64 + tid);
-      {
+      if (tid < 128) {
         const bool g = tid < 64;
         const int l = tid & 63;
         sm.b2[tid] = __ldg((g ? a.sw.g2_b : a.sw.d2_b) + h * 64 + l);
       }
       __syncthreads();
-      {
+      if (tid < 128) {
         // c1[t] = b1[t] + sum_k W1[t][64 + k] C[k]  (context half of the first layer)
         const bool g = tid < 64;
         const int l = tid & 63;
@@ -120,7 +123,7 @@ __global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
       cur_h = h;
     }
 
-    const int base = chunk * 64 + warp * 16;
+    const int base = chunk * kSurrRows + warp * 16;
     if (base >= N) continue;
     const int ra = base + r, rb = base + r + 8;
     const bool va = ra < N, vb = rb < N;
@@ -156,12 +159,13 @@ __global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
       hid[j][1] = pack_bf16x2(gelu_erf(acc[2] + c0), gelu_erf(acc[3] + c1v));
     }
     // Layer 2: the accumulator layout of two adjacent n-tiles is the A-fragment layout
-    // of one 16-wide k-step.
-    float og[8][4], od[8][4];
+    // of one 16-wide k-step.  Output n-tile j of both MLPs is finished and stored before
+    // the next one, so only one tile of each is live.
+    __nv_bfloat16* ya = a.y + ((size_t)ra * H + h) * 64;
+    __nv_bfloat16* yb = a.y + ((size_t)rb * H + h) * 64;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) og[j][i] = od[j][i] = 0.f;
+      float og[4] = {0.f, 0.f, 0.f, 0.f}, od[4] = {0.f, 0.f, 0.f, 0.f};
       const __nv_bfloat16* rowg = &sm.w2[(8 * j + r) * kBStride];
       const __nv_bfloat16* rowd = &sm.w2[(64 + 8 * j + r) * kBStride];
 #pragma unroll
@@ -172,27 +176,22 @@ __global__ void __launch_bounds__(128) surrogate_heads_kernel(HeadAttnArgs a) {
         const uint32_t g1 = *reinterpret_cast<const uint32_t*>(rowg + 16 * kk + 8 + 2 * c);
         const uint32_t d0 = *reinterpret_cast<const uint32_t*>(rowd + 16 * kk + 2 * c);
         const uint32_t d1 = *reinterpret_cast<const uint32_t*>(rowd + 16 * kk + 8 + 2 * c);
-        mma_bf16_16816(og[j], ag, g0, g1);
-        mma_bf16_16816(od[j], ad, d0, d1);
+        mma_bf16_16816(og, ag, g0, g1);
+        mma_bf16_16816(od, ad, d0, d1);
       }
-    }
-    // y = C + sigma(gamma) (.) delta, stored as bf16 in Y[row][h][:].
-    __nv_bfloat16* ya = a.y + ((size_t)ra * H + h) * 64;
-    __nv_bfloat16* yb = a.y + ((size_t)rb * H + h) * 64;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
+      // y = C + sigma(gamma) (.) delta, stored as bf16 in Y[row][h][:].
       const int col = 8 * j + 2 * c;
       const float C0 = sm.ctx[col], C1 = sm.ctx[col + 1];
       const float bg0 = sm.b2[col], bg1 = sm.b2[col + 1];
       const float bd0 = sm.b2[64 + col], bd1 = sm.b2[64 + col + 1];
       if (va)
         *reinterpret_cast<uint32_t*>(ya + col) =
-            pack_bf16x2(C0 + sigmoidf(og[j][0] + bg0) * (od[j][0] + bd0),
-                        C1 + sigmoidf(og[j][1] + bg1) * (od[j][1] + bd1));
+            pack_bf16x2(C0 + sigmoidf(og[0] + bg0) * (od[0] + bd0),
+                        C1 + sigmoidf(og[1] + bg1) * (od[1] + bd1));
       if (vb)
         *reinterpret_cast<uint32_t*>(yb + col) =
-            pack_bf16x2(C0 + sigmoidf(og[j][2] + bg0) * (od[j][2] + bd0),
-                        C1 + sigmoidf(og[j][3] + bg1) * (od[j][3] + bd1));
+            pack_bf16x2(C0 + sigmoidf(og[2] + bg0) * (od[2] + bd0),
+                        C1 + sigmoidf(og[3] + bg1) * (od[3] + bd1));
     }
   }
 }
@@ -209,7 +208,7 @@ cudaError_t launch_mean_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
 cudaError_t launch_surrogate_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
   static_assert(sizeof(SurrSmem) <= 48 * 1024, "surrogate smem fits the default limit");
   prof_before(VP_KERNEL_SURROGATE, st);
-  surrogate_heads_kernel<<<4 * num_sms, 128, sizeof(SurrSmem), st>>>(a);
+  surrogate_heads_kernel<<<4 * num_sms, 32 * kSurrWarps, sizeof(SurrSmem), st>>>(a);
   prof_after(st);
   return cudaGetLastError();
 }

@@ -253,7 +253,7 @@ __global__ void __launch_bounds__(kKeyThreads) router_keys_kernel(RouterArgs a, 
   for (int i = 0; i < 8; ++i) q[i] = __ldcg(sc.q_pool + h * 64 + 8 * part + i) * cscale;
 
   int t0, t1;
-  token_range(N, n_split, split, 32, t0, t1);
+  token_range(N, n_split, split, 128, t0, t1);
   const __nv_bfloat16* kb = a.qkv + (size_t)(H + h) * kHeadDim + 8 * part;
   const __nv_bfloat16* vb = a.qkv + (size_t)(2 * H + h) * kHeadDim + 8 * part;
 
@@ -262,29 +262,30 @@ __global__ void __launch_bounds__(kKeyThreads) router_keys_kernel(RouterArgs a, 
   for (int i = 0; i < 8; ++i) accv[i] = sumv[i] = 0.f;
 
   // The loop bound is uniform across the CTA so that the 8-lane shuffles below always
-  // run with the whole warp; rows past t1 are loaded from row t0 and masked.
-  for (int base = t0; base < t1; base += 64) {
-    const int row = base + g, row2 = base + g + 32;
-    const bool v1 = row < t1, v2 = row2 < t1;
-    const size_t o1 = (size_t)(v1 ? row : t0) * row_pitch, o2 = (size_t)(v2 ? row2 : t0) * row_pitch;
-    const uint4 k1 = __ldg(reinterpret_cast<const uint4*>(kb + o1));
-    const uint4 x1 = __ldg(reinterpret_cast<const uint4*>(vb + o1));
-    const uint4 k2 = __ldg(reinterpret_cast<const uint4*>(kb + o2));
-    const uint4 x2 = __ldg(reinterpret_cast<const uint4*>(vb + o2));
+  // run with the whole warp; rows past t1 are loaded from row t0 and masked.  Four rows per
+  // row group are in flight (eight 16-byte loads per thread) before any arithmetic.
+  for (int base = t0; base < t1; base += 128) {
+    uint4 kr[4], vr[4];
+    bool valid[4];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const bool valid = u ? v2 : v1;
-      const uint4 kk = u ? k2 : k1;
-      const uint4 vv = u ? x2 : x1;
-      const uint32_t kw[4] = {kk.x, kk.y, kk.z, kk.w};
-      const uint32_t vw[4] = {vv.x, vv.y, vv.z, vv.w};
+    for (int u = 0; u < 4; ++u) {
+      const int row = base + g + 32 * u;
+      valid[u] = row < t1;
+      const size_t o = (size_t)(valid[u] ? row : t0) * row_pitch;
+      kr[u] = __ldg(reinterpret_cast<const uint4*>(kb + o));
+      vr[u] = __ldg(reinterpret_cast<const uint4*>(vb + o));
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t kw[4] = {kr[u].x, kr[u].y, kr[u].z, kr[u].w};
+      const uint32_t vw[4] = {vr[u].x, vr[u].y, vr[u].z, vr[u].w};
       float dot = 0.f;
 #pragma unroll
       for (int i = 0; i < 4; ++i) dot += q[2 * i] * bf16_lo(kw[i]) + q[2 * i + 1] * bf16_hi(kw[i]);
       dot += __shfl_xor_sync(0xffffffffu, dot, 1);
       dot += __shfl_xor_sync(0xffffffffu, dot, 2);
       dot += __shfl_xor_sync(0xffffffffu, dot, 4);
-      if (!valid) continue;  // no shuffles below
+      if (!valid[u]) continue;  // no shuffles below
       if (dot > m) {
         const float f = fast_exp2(m - dot);  // 0 when m = -inf
         l *= f;
@@ -493,8 +494,8 @@ cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  int key_split = (2 * num_sms + a.H - 1) / a.H;
-  key_split = max(1, min(min(key_split, kKeySplitMax), (a.N + 127) / 128));
+  int key_split = (4 * num_sms + a.H - 1) / a.H;
+  key_split = max(1, min(min(key_split, kKeySplitMax), (a.N + 255) / 256));
   prof_before(VP_KERNEL_ROUTER_KEYS, st);
   router_keys_kernel<<<dim3(key_split, a.H), kKeyThreads, 0, st>>>(a, sc, key_split);
   prof_after(st);
