@@ -110,6 +110,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
 
+  // Register split (setmaxnreg, per warpgroup): the control warpgroup (warps 0-3) drops to
+  // 80 registers, the two softmax warpgroups rise to 208: 80 x 128 + 208 x 256 = 63,488 <=
+  // 168 x 384, the allocation the CTA is launched with.
+  if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 80;");
+  }
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
@@ -212,6 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax / epilogue
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 208;");
     const int c = (warp - 4) >> 2;  // chain
     const int quarter = warp & 3;   // TMEM lane quarter this warp may access
     const int row_in_tile = quarter * 32 + lane;
