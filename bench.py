@@ -41,6 +41,28 @@ H, d, D = synth.N_HEADS, synth.HEAD_DIM, synth.D_MODEL
 METRIC = "global-attn views/sec, 24-layer MoH global stack at S=100 (518 px, 137,400 tokens)"
 
 
+# ------------------------------------------------------------------ ranks (replicas)
+def replica_seed(base: int, rank: int) -> int:
+    """Each rank runs its own scene (weak scaling): a seed per rank."""
+    return base + 100 * rank
+
+
+def reduce_max_over_ranks(x: float, world: int, device=None) -> float:
+    """The slowest rank's time: the job's time."""
+    if world == 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(ms_per_step: float, world: int, views: int) -> float:
+    """Views per second over the whole job: every rank processes its own S views per step."""
+    return views * world / (ms_per_step / 1e3)
+
+
 def peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -209,7 +231,7 @@ def run_ours(args):
     N, L = WORKLOAD.N, WORKLOAD.layers
     routes = synth.paper_mix_modes(L)
     # Every rank processes its own scene (weak scaling, no data-path collective).
-    seed = WORKLOAD.seed + 100 * rank
+    seed = replica_seed(WORKLOAD.seed, rank)
     host_w = synth.make_stack_weights(seed, L)
     dws = [vpb.to_device(w, dev) for w in host_w]
     layers = [vpb.layer_weights(w) for w in dws]
@@ -246,13 +268,9 @@ def run_ours(args):
     barrier()
     n_launch, per_class_n, per_class_ms = vpb.vp_profile_end()
     clk = clocks.stop()
-    ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max_over_ranks(e0.elapsed_time(e1) / args.steps, world, dev)
     err_bits = vpb.vp_read_device_error(ws)
-    value = WORKLOAD.views * world / (ms / 1e3)
+    value = job_value(ms, world, WORKLOAD.views)
 
     # End to end through the public API: pinned host tokens in, pinned host output out.
     x_host = torch.from_numpy(x_bits.view(np.int16)).view(torch.bfloat16).pin_memory()
@@ -270,11 +288,7 @@ def run_ours(args):
     for _ in range(e2e_steps):
         e2e_step()
     torch.cuda.synchronize()
-    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = reduce_max_over_ranks((time.perf_counter() - t0) * 1e3 / e2e_steps, world, dev)
     finite = bool(torch.isfinite(y_host.float()).all())
 
     # Natural routes of the untrained routers (reported, not used).
@@ -325,7 +339,7 @@ def run_ours(args):
                    "tokens": N, "layers": L, "dim": D, "heads": H, "head_dim": d,
                    "routing": "paper_mix (30 full / 162 surrogate / 192 mean of 384 heads)",
                    "parallelism": f"replicas{world}", "l2": "inputs larger than L2 (281 MB tokens, 1.4 GB workspace)"},
-        "e2e": {"value": WORKLOAD.views * world / (e2e_ms / 1e3), "unit": "views/s",
+        "e2e": {"value": job_value(e2e_ms, world, WORKLOAD.views), "unit": "views/s",
                 "h2d_bytes_per_step": int(x_host.numel() * 2), "d2h_bytes_per_step": int(y_host.numel() * 2),
                 "ms_per_step": e2e_ms},
         "gpu_launches": int(n_launch),

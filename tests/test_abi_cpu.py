@@ -1,0 +1,106 @@
+"""The C ABI without a GPU: the library builds for sm_103a, loads, exports every function
+include/vp.h declares, and rejects bad arguments on the host before touching a device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "vp.h")
+
+
+@pytest.fixture(scope="module")
+def vp():
+    from paper_2609_23733_gb300 import binding, build
+    if not os.path.exists(build.LIB):
+        build.build()
+    return binding
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:vp_status|const char\*)\s+(vp_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("vp_router", "vp_bin_heads", "vp_moh_global_attention", "vp_global_stack",
+                     "vp_workspace_size", "vp_status_string", "vp_head_attention", "vp_linear",
+                     "vp_layer_norm", "vp_router_noalloc"):
+        assert required in names
+
+
+def test_library_exports_every_declared_function(vp):
+    lib = vp.lib()
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(declared_functions()) == set(vp.EXPORTS)
+
+
+def test_status_strings(vp):
+    for code in range(9):
+        assert vp.vp_status_string(code) not in ("", "unknown status")
+    assert vp.vp_status_string(99) == "unknown status"
+
+
+def test_workspace_sizes(vp):
+    small = vp.dims(1044)
+    big = vp.dims(137400)
+    r = vp.vp_workspace_size(small, vp.VP_WS_ROUTER)
+    assert r == vp.vp_workspace_size(big, vp.VP_WS_ROUTER)  # router scratch is independent of N
+    assert vp.vp_workspace_size(big, vp.VP_WS_LAYER) >= r + 137400 * 4 * 1024 * 2
+    assert vp.vp_workspace_size(big, vp.VP_WS_STACK) >= r + 137400 * 5 * 1024 * 2
+    with pytest.raises(vp.VPError) as e:
+        vp.vp_workspace_size(vp.dims(100, d=32), vp.VP_WS_ROUTER)
+    assert e.value.status == 2
+    with pytest.raises(vp.VPError) as e:
+        vp.vp_workspace_size(vp.dims(100, H=33), vp.VP_WS_ROUTER)
+    assert e.value.status == 2
+    with pytest.raises(vp.VPError) as e:
+        vp.vp_workspace_size(small, 7)
+    assert e.value.status == 1
+
+
+def test_host_side_validation(vp):
+    lib = vp.lib()
+    A = 0x10000  # aligned fake device addresses: the checks below fail before any access
+    dm = vp.dims(300)
+    rw = vp.VpRouterWeights(A, A, A, None, None, None)
+    null_rw = vp.VpRouterWeights(None, A, A, None, None, None)
+    bad = vp.dims(300, d=32)
+    # vp_router: missing dims / bad shape / null output / bad alignment / small workspace
+    assert lib.vp_router(None, A, ctypes.byref(rw), None, A, A, None, None, None, None, A, 1 << 30, None) == 1
+    assert lib.vp_router(ctypes.byref(bad), A, ctypes.byref(rw), None, A, A, None, None, None, None, A, 1 << 30, None) == 2
+    assert lib.vp_router(ctypes.byref(dm), A, ctypes.byref(rw), None, None, A, None, None, None, None, A, 1 << 30, None) == 1
+    assert lib.vp_router(ctypes.byref(dm), A + 8, ctypes.byref(rw), None, A, A, None, None, None, None, A, 1 << 30, None) == 3
+    assert lib.vp_router(ctypes.byref(dm), A, ctypes.byref(null_rw), None, A, A, None, None, None, None, A, 1 << 30, None) == 1
+    assert lib.vp_router(ctypes.byref(dm), A, ctypes.byref(rw), None, A, A, None, None, None, None, A, 16, None) == 6
+    # vp_router_noalloc: more heads than its fixed buffer holds
+    assert lib.vp_router_noalloc(ctypes.byref(vp.dims(300, H=33)), A, ctypes.byref(rw), None, A, A,
+                                 None, None, None, None, None) == 8
+    # vp_linear: shapes and alignment
+    assert lib.vp_linear(100, 12, 64, A, A, None, 0, None, None, A, None) == 2
+    assert lib.vp_linear(100, 256, 60, A, A, None, 0, None, None, A, None) == 2
+    assert lib.vp_linear(100, 256, 64, None, A, None, 0, None, None, A, None) == 1
+    assert lib.vp_linear(100, 256, 64, A, A, None, 2, None, None, A, None) == 1
+    assert lib.vp_linear(100, 256, 64, A, A, A + 4, 0, None, None, A, None) == 3
+    # vp_layer_norm: unsupported width
+    assert lib.vp_layer_norm(10, 1000, A, A, A, ctypes.c_float(1e-6), A, None) == 2
+    # vp_bin_heads: no heads
+    assert lib.vp_bin_heads(0, 10, A, A, A, None, None, None) == 2
+    # vp_global_stack: no layers
+    assert lib.vp_global_stack(ctypes.byref(dm), 0, A, None, None, None, None, ctypes.c_float(1e-6), A, 1 << 30, None) == 1
+
+
+def test_valid_call_without_a_gpu_reports_the_device(vp):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    lib = vp.lib()
+    A = 0x10000
+    rw = vp.VpRouterWeights(A, A, A, None, None, None)
+    st = lib.vp_router(ctypes.byref(vp.dims(300)), A, ctypes.byref(rw), None, A, A, None, None, None, None,
+                       A, 1 << 30, None)
+    assert st == 7  # VP_ERR_UNSUPPORTED_DEVICE: nothing was enqueued

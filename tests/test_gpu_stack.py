@@ -1,0 +1,169 @@
+"""GPU parity of Algorithm 1's block stack (vp_global_stack) and the routing-mix sweep at
+full size (S = 64 views, 87,936 tokens) against the float64 oracle.
+
+Stack outputs are the residual stream, stored in bf16 after every block (LayerScale 1
+gives it magnitude > 1), so besides the absolute bar they allow one bf16 step relative to
+the value per block boundary that rounding can cross, and deep stacks use a per-block error
+budget times the depth (see test_stack_24_blocks_s4_natural_routing)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from tests.helpers import BF16_STEP, compare
+
+pytestmark = pytest.mark.gpu
+
+vpb = pytest.importorskip("paper_2609_23733_gb300.binding")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    vpb.lib()
+
+
+def _f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def _run_stack(x_bits, ws_host, N, force=None, H=16):
+    dm = vpb.dims(N, H)
+    dws = [vpb.to_device(w) for w in ws_host]
+    layers = [vpb.layer_weights(w) for w in dws]
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK)
+    x = vpb.bf16_from_bits(x_bits)
+    L = len(ws_host)
+    modes = torch.full((L, H), -1, dtype=torch.int32, device="cuda")
+    s = torch.zeros(L, H, device="cuda")
+    fm = None if force is None else torch.tensor(np.asarray(force, np.int32), device="cuda")
+    vpb.vp_global_stack(dm, x, layers, fm, modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    return _f64(x), modes.cpu().numpy(), s.cpu().numpy()
+
+
+def test_stack_three_blocks_all_modes():
+    N, L = 600, 3
+    g = synth.rng(5)
+    wts = [synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1) for _ in range(L)]
+    for w in wts:
+        w["ls1"] = (0.5 * w["ls1"]).astype(np.float32)
+        w["ls2"] = (0.5 * w["ls2"]).astype(np.float32)
+    x_bits = synth.make_tokens(5, N)
+    force = np.array([synth.forced_mix(16, f) for f in (0.25, 0.5, 1.0)])
+    got, modes, s = _run_stack(x_bits, wts, N, force)
+    want, infos = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w) for w in wts],
+                                      force_modes=force)
+    np.testing.assert_array_equal(modes, force)
+    np.testing.assert_allclose(s[0], infos[0]["s"], rtol=5e-3)
+    compare(got, want, rel=L * BF16_STEP, what="3-block stack")
+
+
+def test_stack_24_blocks_s4_natural_routing():
+    """24 blocks over S=4 views at 224 px (1,044 tokens): untrained routers route every
+    head of every block to mean (saliency ~ 1/N)."""
+    wl = synth.WORKLOADS["s4_layer"]
+    N, L = wl.N, 24
+    wts = synth.make_stack_weights(wl.seed, L)
+    for w in wts:  # keep the residual stream O(1) over 24 blocks
+        w["ls1"] = np.full_like(w["ls1"], 0.2)
+        w["ls2"] = np.full_like(w["ls2"], 0.2)
+    x_bits = synth.make_tokens(wl.seed, N)
+    got, modes, s = _run_stack(x_bits, wts, N)
+    want, infos = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w) for w in wts])
+    np.testing.assert_array_equal(modes, np.array([i["modes"] for i in infos]))
+    assert np.all(modes == synth.MODE_MEAN)
+    # Each block ends in bf16 storage of the residual stream; the two sides round independently
+    # and the differences compound through later blocks, growing about linearly with depth
+    # (measured on GB300: relative norm 2.8e-4 after one block, 6.5e-3 after 24).  The bar is
+    # a per-block budget times the depth: relative norm 5e-4 and mean-abs 4e-4 per block.
+    compare(got, want, max_abs=4e-2, mean_abs=L * 4e-4, rel=4 * BF16_STEP, what="24-block stack")
+    err = np.linalg.norm(got - want) / np.linalg.norm(want)
+    assert err < L * 5e-4, err
+
+
+def test_stack_s32_first_block_sampled_rows_and_view_permutation():
+    """Full size S=32 (43,968 tokens): block 0 against the oracle on sampled rows, and the
+    whole 24-block stack is equivariant under a permutation of the views."""
+    wl = synth.WORKLOADS["s32_stack"]
+    N, P = wl.N, wl.P
+    wts = synth.make_stack_weights(wl.seed, 24)
+    x_bits = synth.make_tokens(wl.seed, N)
+    # Block 0 on the GPU; the oracle recomputes it for sampled rows only (the router and the
+    # mean of V need all rows, every other step is per row).
+    got1, modes1, _ = _run_stack(x_bits, wts[:1], N)
+    lw = oracle.load_layer(wts[0])
+    X = oracle.bf16_bits_to_f64(x_bits)
+    Xt = oracle.round_bf16(oracle.layer_norm(X, lw["ln1_g"], lw["ln1_b"], 1e-6))
+    rows = np.unique(np.concatenate([np.arange(64), np.arange(N - 64, N),
+                                     np.random.default_rng(1).choice(N, 384, replace=False)]))
+    att = oracle.moh_attention(Xt, lw, rows=rows)
+    np.testing.assert_array_equal(modes1[0], att["modes"])
+    Xa = oracle.round_bf16(X[rows] + (att["Y"] @ lw["w_o"].T + lw["b_o"]) * lw["ls1"])
+    Zt = oracle.round_bf16(oracle.layer_norm(Xa, lw["ln2_g"], lw["ln2_b"], 1e-6))
+    Hd = oracle.round_bf16(oracle.gelu(Zt @ lw["w_fc1"].T + lw["b_fc1"]))
+    want1 = oracle.round_bf16(Xa + (Hd @ lw["w_fc2"].T + lw["b_fc2"]) * lw["ls2"])
+    compare(got1[rows], want1, rel=BF16_STEP, what="S=32 block 0 (sampled rows)")
+    # View permutation of the 24-block stack (GPU against GPU).
+    perm = np.random.default_rng(2).permutation(wl.views)
+    xp_bits = x_bits.reshape(wl.views, P, -1)[perm].reshape(N, -1)
+    out, modes, _ = _run_stack(x_bits, wts, N)
+    outp, modesp, _ = _run_stack(xp_bits, wts, N)
+    np.testing.assert_array_equal(modes, modesp)
+    assert np.all(np.isfinite(out))
+    ref = out.reshape(wl.views, P, -1)[perm].reshape(N, -1)
+    rel = np.linalg.norm(outp - ref) / np.linalg.norm(ref)
+    assert rel < 1e-2, rel
+
+
+@pytest.mark.parametrize("frac", [0.0, 0.25, 0.5, 1.0])
+def test_mix_sweep_s64_sampled_rows(frac, _s64_case):
+    """Single layer at S=64 views (87,936 tokens) with 0 / 25 / 50 / 100 % of the heads
+    forced to full mode; every head checked on sampled rows against the oracle."""
+    x_bits, w, lw, qkv, routers, rows = _s64_case
+    N, H = qkv.shape[0], 16
+    force = synth.forced_mix(H, frac)
+    dm = vpb.dims(N, H)
+    dw = vpb.to_device(w)
+    ws = vpb.workspace(dm, vpb.VP_WS_LAYER)
+    out = torch.zeros(N, H * 64, dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros(N, H * 64, dtype=torch.bfloat16, device="cuda")
+    modes = torch.zeros(H, dtype=torch.int32, device="cuda")
+    vpb.vp_moh_global_attention(dm, vpb.bf16_from_bits(x_bits), dw["w_qkv"], dw["b_qkv"], dw["w_o"], dw["b_o"],
+                                vpb.router_weights(dw), vpb.surrogate_weights(dw),
+                                torch.from_numpy(force).cuda(), out, None, y, None, modes, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    np.testing.assert_array_equal(modes.cpu().numpy(), force)
+    Y = np.zeros((len(rows), H, 64))
+    for h in range(H):
+        Q, K, V = qkv[:, 0, h], qkv[:, 1, h], qkv[:, 2, h]
+        r = routers[h]
+        if force[h] == synth.MODE_FULL:
+            Y[:, h] = oracle.full_attention(Q, K, V, rows=rows)
+        elif force[h] == synth.MODE_SURROGATE:
+            mg = (lw["s_g1_w"][h], lw["s_g1_b"][h], lw["s_g2_w"][h], lw["s_g2_b"][h])
+            md = (lw["s_d1_w"][h], lw["s_d1_b"][h], lw["s_d2_w"][h], lw["s_d2_b"][h])
+            Y[:, h], _ = oracle.surrogate_attention(V, r, mg, md, rows=rows)
+        else:
+            Y[:, h], _ = oracle.mean_pooling(V, n_rows=len(rows))
+    Y = oracle.round_bf16(Y.reshape(len(rows), -1))
+    compare(_f64(y)[rows], Y, what=f"Y at {frac:.0%} full")
+    compare(_f64(out)[rows], oracle.round_bf16(Y @ lw["w_o"].T + lw["b_o"]), what=f"out at {frac:.0%} full")
+
+
+@pytest.fixture(scope="module")
+def _s64_case():
+    wl = synth.WORKLOADS["s64_mix_sweep"]
+    N = wl.N
+    w = synth.make_layer_weights(synth.rng(wl.seed), bias_std=0.02)
+    x_bits = synth.make_tokens(wl.seed, N)
+    lw = oracle.load_layer(w)
+    qkv = oracle.qkv_projection(oracle.bf16_bits_to_f64(x_bits), lw)
+    routers = [oracle.layer.head_router(qkv[:, 0, h], qkv[:, 1, h], lw, h)[2] for h in range(16)]
+    rows = np.unique(np.concatenate([np.arange(0, 130), np.arange(N - 130, N),
+                                     np.random.default_rng(3).choice(N, 256, replace=False)]))
+    return x_bits, w, lw, qkv, routers, rows
