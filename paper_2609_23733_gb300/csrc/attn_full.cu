@@ -252,11 +252,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Row max: eight independent 3-input max chains, then a short tree.
         float mx;
         {
+          // Chain k covers s[k + 8 i], i = 0..15: one 2-input max, then seven 3-input ones.
           float t[8];
 #pragma unroll
-          for (int k = 0; k < 8; ++k) t[k] = s[k];
+          for (int k = 0; k < 8; ++k) t[k] = fmaxf(s[k], s[8 + k]);
 #pragma unroll
-          for (int i = 8; i < 128; i += 16) {
+          for (int i = 16; i < 128; i += 16) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) t[k] = fmax3(t[k], s[i + k], s[i + 8 + k]);
           }
