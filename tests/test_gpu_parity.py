@@ -233,6 +233,24 @@ def test_head_modes_match_oracle(N):
         compare(got[:, h], oracle.round_bf16(want[:, h]), what=f"head {h} mode {modes[h]}")
 
 
+@pytest.mark.parametrize("N", [5000, 9999])
+def test_full_attention_many_items(N):
+    # More (head, query pair) work items than CTAs: every CTA runs several items in turn and
+    # reuses its TMEM, barriers and pipeline stages across them.
+    H = 16
+    g = np.random.default_rng(N)
+    qkv = g.standard_normal((N, 3, H, 64)).astype(np.float32)
+    qkv_bits = synth.f32_to_bf16_bits(qkv)
+    w = synth.make_layer_weights(synth.rng(1), D=H * 64, H=H)
+    q = oracle.bf16_bits_to_f64(qkv_bits).reshape(N, 3, H, 64)
+    got = _run_heads(qkv_bits, w, N, H, np.full(H, 2, np.int32), np.zeros((H, 64)), np.zeros((H, 64)))
+    rows = np.unique(np.concatenate([np.arange(0, 300), np.arange(N - 300, N),
+                                     np.random.default_rng(0).choice(N, 400, replace=False)]))
+    for h in range(H):
+        want = oracle.full_attention(q[:, 0, h], q[:, 1, h], q[:, 2, h], rows=rows)
+        compare(got[rows, h], oracle.round_bf16(want), what=f"split head {h}")
+
+
 def test_full_attention_peaked_scores():
     # Large logits make the running max move late in the key sweep (lazy rescaling path).
     N, H = 1000, 2
