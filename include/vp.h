@@ -247,8 +247,9 @@ vp_status vp_router_noalloc(const vp_dims* dims, const vp_bf16* qkv, const vp_ro
 #define VP_KERNEL_ROUTER_KEYS 2
 #define VP_KERNEL_ROUTER_R 3
 #define VP_KERNEL_BIN_HEADS 4
-#define VP_KERNEL_ATTN_FULL 5
-#define VP_KERNEL_SURROGATE 6
+#define VP_KERNEL_ATTN_FULL 5   /* all heads of a layer: full-attention kernel + cheap-heads
+                                   kernel overlapping its tail, timed as one bracket */
+#define VP_KERNEL_SURROGATE 6   /* (unused: surrogate and mean heads are timed with class 5) */
 #define VP_KERNEL_MEAN 7
 #define VP_KERNEL_LAYER_NORM 8
 #define VP_KERNEL_CLASSES 9

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libvp.so")
-SOURCES = ["api.cu", "router.cu", "modes.cu", "attn_full.cu", "gemm.cu", "layernorm.cu",
+SOURCES = ["api.cu", "router.cu", "attn_full.cu", "heads_cheap.cu", "gemm.cu", "layernorm.cu",
            "router_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -78,6 +78,10 @@ void prof_before(int kind, cudaStream_t st) {
   }
 }
 
+void prof_extra_launch() {
+  if (g_prof.active) ++g_prof.launches;
+}
+
 void prof_after(cudaStream_t st) {
   Profiler& p = g_prof;
   if (!p.active || !p.pending) return;
@@ -212,7 +216,7 @@ SurrogateArgs make_surrogate_args(const vp_surrogate_weights* sw) {
 // Runs the three mode kernels for bins already in device memory.
 vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* head_ids,
                     const int32_t* offsets, const float* ctx, const float* mean_v,
-                    const vp_surrogate_weights* sw, __nv_bfloat16* y, unsigned int* err,
+                    const vp_surrogate_weights* sw, __nv_bfloat16* y, const RouterScratch& sc,
                     cudaStream_t st) {
   HeadAttnArgs ha{};
   ha.N = dm->N;
@@ -224,12 +228,9 @@ vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* 
   ha.mean_v = mean_v;
   ha.sw = make_surrogate_args(sw);
   ha.y = y;
-  ha.err = err;
-  const int sms = device_sm_count();
-  VP_TRY(from_cuda(launch_full_heads(ha, sms, st)));
-  VP_TRY(from_cuda(launch_surrogate_heads(ha, sms, st)));
-  VP_TRY(from_cuda(launch_mean_heads(ha, sms, st)));
-  return VP_OK;
+  ha.err = sc.err;
+  ha.cheap_counter = sc.cheap_counter;
+  return from_cuda(launch_heads(ha, device_sm_count(), st));
 }
 
 // QKV projection -> router -> bins -> heads -> W_O (+ optional LayerScale / residual).
@@ -256,7 +257,7 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
   ra.s_out = s_out;
   ra.modes_out = modes_out;
   VP_TRY(from_cuda(launch_router(ra, sc, sms, st)));
-  VP_TRY(run_heads(dm, qkv, sc.head_ids, sc.offsets, sc.ctx, sc.mean_v, sw, y, sc.err, st));
+  VP_TRY(run_heads(dm, qkv, sc.head_ids, sc.offsets, sc.ctx, sc.mean_v, sw, y, sc, st));
   LinearArgs lo{};
   lo.M = N;
   lo.N = D;
@@ -407,7 +408,7 @@ vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32
   VP_TRY(check_device());
   RouterScratch sc = carve_router_scratch(ws, dims->H);
   return run_heads(dims, reinterpret_cast<const __nv_bfloat16*>(qkv), head_ids, offsets, ctx,
-                   mean_v, sw, reinterpret_cast<__nv_bfloat16*>(y), sc.err,
+                   mean_v, sw, reinterpret_cast<__nv_bfloat16*>(y), sc,
                    static_cast<cudaStream_t>(stream));
 }
 

@@ -18,6 +18,9 @@
 // products, and S_c(j+1) is issued as soon as chain c has read S_c(j).
 // TMEM: S_0 [0,128) S_1 [128,256) O_0 [256,320) O_1 [320,384) P_0 [384,448) P_1 [448,512).
 // Keys past N are zero-filled by TMA and masked to -inf; query rows past N are not stored.
+// Every CTA signals its dependents at once (griddepcontrol.launch_dependents), so the
+// cheap-heads kernel queued behind this one (heads_cheap.cu) can take the SMs that the last
+// full-attention round leaves idle.
 // Every mbarrier wait is bounded (mbar_wait); on timeout the CTA records the error, stops
 // issuing work, waits (bounded) for its own outstanding copies and MMAs, frees TMEM, exits.
 #include <math.h>
@@ -79,6 +82,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = warp_id(), lane = lane_id();
   volatile int* abort_flag = &sm.abort_flag;
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
@@ -365,9 +369,7 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
   e = cudaFuncSetAttribute(attn_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.err};
-  prof_before(VP_KERNEL_ATTN_FULL, st);
   attn_full_kernel<<<num_sms, kThreads, smem, st>>>(tmap, prm);
-  prof_after(st);
   return cudaGetLastError();
 }
 

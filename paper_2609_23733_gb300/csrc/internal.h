@@ -34,6 +34,7 @@ struct RouterScratch {
   float* mean_v;                // [H][64]
   int32_t* head_ids;            // [H]
   int32_t* offsets;             // [4]
+  unsigned int* cheap_counter;  // work counter of the cheap head modes
 };
 
 size_t router_scratch_bytes(int H);
@@ -81,11 +82,14 @@ struct HeadAttnArgs {
   SurrogateArgs sw;
   __nv_bfloat16* y;
   unsigned int* err;
+  unsigned int* cheap_counter;  // one word of scratch, zeroed by the launcher
 };
 
-cudaError_t launch_mean_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
-cudaError_t launch_surrogate_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+// Full-mode heads (attn_full.cu).
 cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+// All heads of a layer: full-mode heads, then surrogate and mean heads overlapped with the
+// full-attention tail (heads_cheap.cu).
+cudaError_t launch_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
 
 struct LinearArgs {
   int M, N, K;
@@ -113,6 +117,7 @@ cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols,
 // Launch profiler hooks (no-ops unless vp_profile_begin is active).
 void prof_before(int kind, cudaStream_t st);
 void prof_after(cudaStream_t st);
+void prof_extra_launch();  // one more kernel inside the current bracket
 
 int device_sm_count();
 bool device_is_sm103();

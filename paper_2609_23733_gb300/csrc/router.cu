@@ -479,6 +479,7 @@ RouterScratch carve_router_scratch(void* ws, int H) {
   p += kMaxHeads * 4;
   sc.head_ids = reinterpret_cast<int32_t*>(p);
   sc.offsets = sc.head_ids + kMaxHeads;
+  sc.cheap_counter = sc.counters + 96;  // counters[0 .. 2 * kMaxHeads] serve the router
   return sc;
 }
 
