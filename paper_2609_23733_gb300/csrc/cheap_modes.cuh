@@ -34,10 +34,6 @@ __device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, uint
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ float gelu_erf(float x) {
-  return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
-}
-
 __device__ __forceinline__ float sigmoidf(float x) { return 1.f / (1.f + __expf(-x)); }
 
 struct SurrSmem {
@@ -137,8 +133,8 @@ __device__ __forceinline__ void surrogate_rows(const HeadAttnArgs& a, const Surr
     }
     const int col = 8 * j + 2 * c;
     const float c0 = sm.c1[col], c1v = sm.c1[col + 1];
-    hid[j][0] = pack_bf16x2(gelu_erf(acc[0] + c0), gelu_erf(acc[1] + c1v));
-    hid[j][1] = pack_bf16x2(gelu_erf(acc[2] + c0), gelu_erf(acc[3] + c1v));
+    hid[j][0] = pack_bf16x2(gelu_as(acc[0] + c0), gelu_as(acc[1] + c1v));
+    hid[j][1] = pack_bf16x2(gelu_as(acc[2] + c0), gelu_as(acc[3] + c1v));
   }
   // Layer 2: the accumulator layout of two adjacent n-tiles is the A-fragment layout of one
   // 16-wide k-step.  Output n-tile j of both MLPs is finished and stored before the next.

@@ -288,6 +288,28 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// erf(x) by Abramowitz & Stegun, Handbook of Mathematical Functions (1964), formula 7.1.26:
+// erf(|x|) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-x^2), t = 1 / (1 + p |x|),
+// absolute error <= 1.5e-7 (the book's bound), odd in x.  Two MUFU operations (reciprocal,
+// 2^x) and seven FMA-pipe operations.
+__device__ __forceinline__ float erf_as(float x) {
+  const float ax = fabsf(x);
+  float t;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t) : "f"(fmaf(0.3275911f, ax, 1.f)));
+  float poly = fmaf(t, 1.061405429f, -1.453152027f);
+  poly = fmaf(t, poly, 1.421413741f);
+  poly = fmaf(t, poly, -0.284496736f);
+  poly = fmaf(t, poly, 0.254829592f);
+  poly *= t;
+  const float e = fast_exp2(-1.4426950408889634f * ax * ax);
+  return copysignf(fmaf(-poly, e, 1.f), x);
+}
+
+// GELU, erf form: 0.5 x (1 + erf(x / sqrt 2)).
+__device__ __forceinline__ float gelu_as(float x) {
+  return 0.5f * x * (1.f + erf_as(x * 0.70710678118654752f));
+}
+
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 

@@ -45,10 +45,6 @@ struct GemmParams {
   unsigned int* err;
 };
 
-__device__ __forceinline__ float gelu_erf(float x) {
-  return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
-}
-
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
                 const __grid_constant__ CUtensorMap tmap_b,
@@ -186,7 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (prm.act == VP_ACT_GELU) {
 #pragma unroll
-            for (int k = 0; k < 32; ++k) x[k] = gelu_erf(x[k]);
+            for (int k = 0; k < 32; ++k) x[k] = gelu_as(x[k]);
           }
           if (prm.scale) {
 #pragma unroll

@@ -60,6 +60,19 @@ def test_linear_matches_oracle(M, N, K, act, with_bias, with_scale, with_res):
     compare(_f64(out), oracle.round_bf16(ref), rel=BF16_STEP if with_res else 0.0, what="linear")
 
 
+def test_gemm_gelu_epilogue_is_exact_to_bf16():
+    # out = GELU(x) through an identity weight: the epilogue's erf (A&S 7.1.26, |error| <=
+    # 1.5e-7) must give the exact GELU to within one bf16 rounding step.
+    K = 256
+    x = oracle.round_bf16(np.linspace(-6.0, 6.0, 300 * K).reshape(300, K))
+    out = vpb.vp_linear(_bf(x), _bf(np.eye(K)), None, 1)
+    torch.cuda.synchronize()
+    want = oracle.gelu(x)
+    got = _f64(out)
+    # One bf16 step relative, plus the absolute error of the erf approximation (0.5 |x| 1.5e-7).
+    assert np.all(np.abs(got - want) <= 2.0 ** -8 * np.abs(want) + 5e-7)
+
+
 def test_linear_residual_in_place():
     g = np.random.default_rng(5)
     A = oracle.round_bf16(g.standard_normal((260, 512)))

@@ -89,8 +89,11 @@ def test_stack_s32_first_block_sampled_rows_and_view_permutation():
     """Full size S=32 (43,968 tokens): block 0 against the oracle on sampled rows, and the
     whole 24-block stack is equivariant under a permutation of the views."""
     wl = synth.WORKLOADS["s32_stack"]
-    N, P = wl.N, wl.P
-    wts = synth.make_stack_weights(wl.seed, 24)
+    N, P, L = wl.N, wl.P, 24
+    wts = synth.make_stack_weights(wl.seed, L)
+    for w in wts:  # keep the residual stream O(1) over 24 blocks
+        w["ls1"] = np.full_like(w["ls1"], 0.2)
+        w["ls2"] = np.full_like(w["ls2"], 0.2)
     x_bits = synth.make_tokens(wl.seed, N)
     # Block 0 on the GPU; the oracle recomputes it for sampled rows only (the router and the
     # mean of V need all rows, every other step is per row).
@@ -115,8 +118,10 @@ def test_stack_s32_first_block_sampled_rows_and_view_permutation():
     np.testing.assert_array_equal(modes, modesp)
     assert np.all(np.isfinite(out))
     ref = out.reshape(wl.views, P, -1)[perm].reshape(N, -1)
+    # Exact in real arithmetic; numerically the router's and the mean heads' token sums run in
+    # another order, and the differences compound like the stack's rounding (same budget).
     rel = np.linalg.norm(outp - ref) / np.linalg.norm(ref)
-    assert rel < 1e-2, rel
+    assert rel < L * 5e-4, rel
 
 
 @pytest.mark.parametrize("frac", [0.0, 0.25, 0.5, 1.0])
