@@ -376,9 +376,46 @@ def run_ours(args):
     }
     if args.full_layer:
         line["full_attention_s100"] = full_attention_probe(vpb, dev, N, dws[0], pk)
+    if args.s32:
+        line["stack_s32"] = s32_probe(vpb, dev)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
+
+
+def s32_probe(vpb, dev, steps=3, warmup=2):
+    """The 24-layer stack at S=32 views (518 px, 43,968 tokens) with the untrained routers
+    deciding the routes (the second stack configuration of the metric)."""
+    import torch
+    wl = synth.WORKLOADS["s32_stack"]
+    N = wl.N
+    dws = [vpb.to_device(w, dev) for w in synth.make_stack_weights(wl.seed, wl.layers)]
+    layers = [vpb.layer_weights(w) for w in dws]
+    x0 = vpb.bf16_from_bits(synth.make_tokens(wl.seed, N), dev)
+    x = torch.empty_like(x0)
+    modes = torch.zeros(wl.layers, H, dtype=torch.int32, device=dev)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK, dev)
+
+    def step():
+        x.copy_(x0)
+        vpb.vp_global_stack(dm, x, layers, None, modes, None, 1e-6, ws)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    m = modes.cpu().numpy()
+    return {"workload": wl.name, "views": wl.views, "tokens": N, "layers": wl.layers,
+            "routing": "natural (untrained routers)", "ms_per_forward": ms,
+            "views_per_s": wl.views / (ms / 1e3),
+            "routes": {"mean": int((m == 0).sum()), "surrogate": int((m == 1).sum()), "full": int((m == 2).sum())}}
 
 
 def full_attention_probe(vpb, dev, N, dw, pk):
@@ -483,6 +520,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--full-layer", action="store_true", default=True)
     ap.add_argument("--no-full-layer", dest="full_layer", action="store_false")
+    ap.add_argument("--s32", action="store_true", default=True)
+    ap.add_argument("--no-s32", dest="s32", action="store_false")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "layer_norm", "router", "surrogate"],
                     default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
