@@ -5,7 +5,7 @@
 // read from the device bins.  The two query tiles of an item run as two independent
 // chains, c = 0 and c = 1, that share the K/V pipeline:
 //   warp 0        TMA producer: both Q tiles once per item, K/V tiles through a 4-stage ring.
-//   warp 1        TMEM owner.  Warps 1 and 2: one lane each issues chain c's tcgen05.mma:
+//   warp 1        TMEM owner.  Warps 1 and 2: one elected lane each issues chain c's tcgen05.mma:
 //                 S_c = Q_c K^T (SS form, 128 x 128 fp32 in TMEM) and O_c += P_c V
 //                 (TS form: P_c read from TMEM as bf16, V from shared memory, MN-major).
 //   warps 4-7     softmax of chain 0, warps 8-11 softmax of chain 1: one query row per
@@ -60,12 +60,6 @@ struct FullParams {
   unsigned int* err;
 };
 
-__device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity, unsigned int* err,
-                                         volatile int* abort_flag) {
-  const bool ok = mbar_wait(bar, parity, err, abort_flag);
-  return __all_sync(0xffffffffu, ok);  // TMEM access below is warp-collective
-}
-
 __global__ void __launch_bounds__(kThreads, 1)
     attn_full_kernel(const __grid_constant__ CUtensorMap tmap_qkv, FullParams prm) {
   extern __shared__ unsigned char smem_raw[];
@@ -80,7 +74,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int items = n_heads * n_pairs;
   if ((int)blockIdx.x >= items) return;  // uniform across the CTA
 
-  const int warp = warp_id(), lane = lane_id();
+  const int warp = warp_uniform_id(), lane = lane_id();
   volatile int* abort_flag = &sm.abort_flag;
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
@@ -112,7 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = sm.tmem_base;
+  const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
 
   // Register split (setmaxnreg, per warpgroup): the control warpgroup (warps 0-3) drops to
   // 80 registers, the two softmax warpgroups rise to 208: 80 x 128 + 208 x 256 = 63,488 <=
@@ -122,89 +116,100 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      uint32_t lc = 0, ic = 0;
-      bool ok = true;
-      for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
-        const int h = __ldg(prm.head_ids + first + item / n_pairs);
-        const int qp = item % n_pairs;
-        ok = mbar_wait(&sm.q_empty, (ic & 1) ^ 1, prm.err, abort_flag);
-        if (!ok) break;
+    // The whole warp walks the loop (so that coordinates and addresses stay warp-uniform);
+    // one elected lane issues the copies.
+    uint32_t lc = 0, ic = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
+      const int h = __shfl_sync(0xffffffffu, __ldg(prm.head_ids + first + item / n_pairs), 0);
+      const int qp = item % n_pairs;
+      ok = mbar_wait_warp(&sm.q_empty, (ic & 1) ^ 1, prm.err, abort_flag);
+      if (!ok) break;
+      if (elect_one()) {
         mbar_arrive_expect_tx(&sm.q_full, 2 * kTileBytes);
         tma_load_2d(sm.q[0], &tmap_qkv, &sm.q_full, h * 64, qp * 2 * kBM);
         tma_load_2d(sm.q[1], &tmap_qkv, &sm.q_full, h * 64, qp * 2 * kBM + kBM);
-        for (int j = 0; j < n_kv; ++j, ++lc) {
-          const int st = lc % kStages;
-          ok = mbar_wait(&sm.kv_empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
-          if (!ok) break;
+      }
+      __syncwarp();
+      for (int j = 0; j < n_kv; ++j, ++lc) {
+        const int st = lc % kStages;
+        ok = mbar_wait_warp(&sm.kv_empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
+        if (!ok) break;
+        if (elect_one()) {
           mbar_arrive_expect_tx(&sm.k_full[st], kTileBytes);
           tma_load_2d(sm.k[st], &tmap_qkv, &sm.k_full[st], (H + h) * 64, j * kBN);
           mbar_arrive_expect_tx(&sm.v_full[st], kTileBytes);
           tma_load_2d(sm.v[st], &tmap_qkv, &sm.v_full[st], (2 * H + h) * 64, j * kBN);
         }
+        __syncwarp();
       }
-      if (!ok) {
-        // Let the copies this thread issued land before the CTA releases its smem.
-        // ic counts items whose Q load was issued when the loop broke inside the K/V loop,
-        // and items + 1 when it broke at the Q wait; waiting on the last issued phase is
-        // bounded either way.
-        if (ic > 0)
-          for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.q_full, (ic - 1) & 1); ++t) {}
-        for (int s = 0; s < kStages; ++s) {
-          if (lc > (uint32_t)s) {
-            const uint32_t last = (lc - 1 - s) / kStages * kStages + s;  // last use of stage s
-            const uint32_t par = (last / kStages) & 1;
-            for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.k_full[s], par); ++t) {}
-            for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.v_full[s], par); ++t) {}
-          }
+    }
+    if (!ok && lane == 0) {
+      // Let the copies this warp issued land before the CTA releases its smem.
+      // ic counts items whose Q load was issued when the loop broke inside the K/V loop,
+      // and items + 1 when it broke at the Q wait; waiting on the last issued phase is
+      // bounded either way.
+      if (ic > 0)
+        for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.q_full, (ic - 1) & 1); ++t) {}
+      for (int s = 0; s < kStages; ++s) {
+        if (lc > (uint32_t)s) {
+          const uint32_t last = (lc - 1 - s) / kStages * kStages + s;  // last use of stage s
+          const uint32_t par = (last / kStages) & 1;
+          for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.k_full[s], par); ++t) {}
+          for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.v_full[s], par); ++t) {}
         }
       }
     }
   } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------ MMA issuers (chain c)
+    // Converged warp; the elected lane (the same lane every time: elect.sync picks the
+    // lowest active lane) issues the MMAs and the commits that track them.
     const int c = warp - 1;
-    if (lane == 0) {
-      const uint32_t id_s = idesc_bf16(kBM, kBN, 0, 0);  // Q (K-major) x K^T (K-major)
-      const uint32_t id_o = idesc_bf16(kBM, 64, 0, 1);   // P (TMEM) x V (MN-major)
-      const uint64_t dq = sdesc_sw128(smem_u32(sm.q[c]));
-      const uint32_t t_s = tmem + kColS + c * kBN;
-      const uint32_t t_o = tmem + kColO + c * 64;
-      const uint32_t t_p = tmem + kColP + c * 64;
-      uint32_t lc = 0, ic = 0, g = 0;  // K/V tiles seen, items, S/P/O tiles of this chain
-      bool ok = true;
-      for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
-        ok = mbar_wait(&sm.q_full, ic & 1, prm.err, abort_flag);
-        if (!ok) break;
+    const uint32_t id_s = idesc_bf16(kBM, kBN, 0, 0);  // Q (K-major) x K^T (K-major)
+    const uint32_t id_o = idesc_bf16(kBM, 64, 0, 1);   // P (TMEM) x V (MN-major)
+    const uint64_t dq = sdesc_sw128(smem_u32(sm.q[c]));
+    const uint32_t t_s = tmem + kColS + c * kBN;
+    const uint32_t t_o = tmem + kColO + c * 64;
+    const uint32_t t_p = tmem + kColP + c * 64;
+    uint32_t lc = 0, ic = 0, g = 0;  // K/V tiles seen, items, S/P/O tiles of this chain
+    bool ok = true;
+    for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
+      ok = mbar_wait_warp(&sm.q_full, ic & 1, prm.err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t lc0 = lc, g0 = g;
+      auto issue_s = [&](int j) -> bool {
+        const uint32_t l = lc0 + j, gg = g0 + j;
+        const int st = l % kStages;
+        if (!mbar_wait_warp(&sm.k_full[st], (l / kStages) & 1, prm.err, abort_flag)) return false;
+        if (!mbar_wait_warp(&sm.s_empty[c], (gg & 1) ^ 1, prm.err, abort_flag)) return false;
         tc_fence_after();
-        const uint32_t lc0 = lc, g0 = g;
-        auto issue_s = [&](int j) -> bool {
-          const uint32_t l = lc0 + j, gg = g0 + j;
-          const int st = l % kStages;
-          if (!mbar_wait(&sm.k_full[st], (l / kStages) & 1, prm.err, abort_flag)) return false;
-          if (!mbar_wait(&sm.s_empty[c], (gg & 1) ^ 1, prm.err, abort_flag)) return false;
-          tc_fence_after();
-          const uint64_t dk = sdesc_sw128(smem_u32(sm.k[st]));
+        const uint64_t dk = sdesc_sw128(smem_u32(sm.k[st]));
+        if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)  // 4 x K=16 covers d = 64 (+32 bytes per step)
             tc_mma_ss(t_s, dq + 2 * kk, dk + 2 * kk, id_s, kk > 0);
           tc_commit(&sm.s_full[c]);
           if (j == n_kv - 1) tc_commit(&sm.q_empty);
-          return true;
-        };
-        ok = issue_s(0);
-        for (int j = 0; j < n_kv && ok; ++j) {
-          if (j + 1 < n_kv) {
-            ok = issue_s(j + 1);  // as soon as the softmax has read S_c(j)
-            if (!ok) break;
-          }
-          const uint32_t l = lc0 + j, gg = g0 + j;
-          const int st = l % kStages;
-          ok = mbar_wait(&sm.p_full[c], gg & 1, prm.err, abort_flag) &&
-               mbar_wait(&sm.v_full[st], (l / kStages) & 1, prm.err, abort_flag) &&
-               (j > 0 || mbar_wait(&sm.o_empty[c], (ic & 1) ^ 1, prm.err, abort_flag));
+        }
+        __syncwarp();
+        return true;
+      };
+      ok = issue_s(0);
+      for (int j = 0; j < n_kv && ok; ++j) {
+        if (j + 1 < n_kv) {
+          ok = issue_s(j + 1);  // as soon as the softmax has read S_c(j)
           if (!ok) break;
-          tc_fence_after();
-          const uint64_t dv = sdesc_sw128(smem_u32(sm.v[st]));
+        }
+        const uint32_t l = lc0 + j, gg = g0 + j;
+        const int st = l % kStages;
+        ok = mbar_wait_warp(&sm.p_full[c], gg & 1, prm.err, abort_flag) &&
+             mbar_wait_warp(&sm.v_full[st], (l / kStages) & 1, prm.err, abort_flag) &&
+             (j > 0 || mbar_wait_warp(&sm.o_empty[c], (ic & 1) ^ 1, prm.err, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        const uint64_t dv = sdesc_sw128(smem_u32(sm.v[st]));
+        if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk)  // 8 x K=16 covers 128 keys: 8 TMEM columns, 2 KB of V
             tc_mma_ts(t_o, t_p + 8 * kk, dv + (uint64_t)(kk * 128), id_o,
@@ -212,13 +217,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_commit(&sm.o_bar[c]);
           tc_commit(&sm.kv_empty[st]);
         }
-        lc = lc0 + n_kv;
-        g = g0 + n_kv;
+        __syncwarp();
       }
-      if (!ok) {
+      lc = lc0 + n_kv;
+      g = g0 + n_kv;
+    }
+    if (!ok) {
+      if (elect_one()) {
         tc_commit(&sm.drain[c]);
         for (int t = 0; t < 1000000 && !mbar_try_wait(&sm.drain[c], 0); ++t) {}
       }
+      __syncwarp();
     }
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax / epilogue
@@ -239,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qp = item % n_pairs;
       float m = 0.f, lsum = 0.f;
       for (int j = 0; j < n_kv; ++j, ++g) {
-        ok = wait_all(&sm.s_full[c], g & 1, prm.err, abort_flag);
+        ok = mbar_wait_warp(&sm.s_full[c], g & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
         float s[128];
@@ -277,16 +286,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           alpha = fast_exp2(m - mx2);
           m = mx2;
         }
-        // p = 2^(s cs - m), summed in packed pairs.
+        // p = 2^(s cs - m), summed in packed pairs and packed to bf16 pairs for P (before the
+        // wait for P_c(g-1) V below, so that only the TMEM stores follow it).
         const float2 c2 = make_float2(cs, cs), nm = make_float2(-m, -m);
         float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+        uint32_t pk[64];
 #pragma unroll
         for (int i = 0; i < 64; ++i) {
           float2 x = ffma2(make_float2(s[2 * i], s[2 * i + 1]), c2, nm);
           x.x = fast_exp2(x.x);
           x.y = fast_exp2(x.y);
-          s[2 * i] = x.x;
-          s[2 * i + 1] = x.y;
+          pk[i] = pack_bf16x2(x.x, x.y);
           if (i & 1)
             acc1 = fadd2(acc1, x);
           else
@@ -296,17 +306,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         lsum = lsum * alpha + (at.x + at.y);
         // P_c and O_c are free once P_c(g-1) V has completed.
         if (g > 0) {
-          ok = wait_all(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
+          ok = mbar_wait_warp(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
           if (!ok) break;
           tc_fence_after();
         }
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) {
-          uint32_t pk[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(s[32 * cc + 2 * i], s[32 * cc + 2 * i + 1]);
-          tmem_st16(t_p + 16 * cc, pk);
-        }
+        for (int cc = 0; cc < 4; ++cc) tmem_st16(t_p + 16 * cc, pk + 16 * cc);
         if (__any_sync(0xffffffffu, need)) {
           float o[64];
           tmem_ld32(t_o, o);
@@ -323,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
       // Epilogue: O / sum -> bf16 -> Y[row][h][:]
-      ok = wait_all(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
+      ok = mbar_wait_warp(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
       float o[64];

@@ -81,6 +81,14 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsign
   }
 }
 
+// mbar_wait for a converged warp: every lane polls, and the result is the same on every lane
+// (TMEM accesses and elected-lane issue after it are warp-collective).
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, unsigned int* err,
+                                               volatile int* abort_flag) {
+  const bool ok = mbar_wait(bar, parity, err, abort_flag);
+  return __all_sync(0xffffffffu, ok);
+}
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const void* tmap) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
@@ -312,5 +320,26 @@ __device__ __forceinline__ float gelu_as(float x) {
 
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
+
+// The warp index as a value the compiler can prove is the same on every lane (a shuffle
+// from lane 0).  Operands of tcgen05 and TMA instructions live in uniform registers; values
+// derived from this index stay there, where values derived from threadIdx.x would have to be
+// moved (and checked for uniformity) at every such instruction.
+__device__ __forceinline__ int warp_uniform_id() {
+  return __shfl_sync(0xffffffffu, (int)(threadIdx.x >> 5), 0);
+}
+
+// True on exactly one lane of a converged warp (elect.sync): that lane issues the warp's
+// single-thread instructions (tcgen05.mma, tcgen05.commit, TMA copies) while the loop around
+// them, and every operand, stays warp-uniform.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "elect.sync _|p, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(pred));
+  return pred != 0;
+}
 
 }  // namespace vp

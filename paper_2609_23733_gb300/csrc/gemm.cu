@@ -57,7 +57,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tiles = m_tiles * n_tiles;
   const int k_blocks = (K + kBK - 1) / kBK;
   if ((int)blockIdx.x >= tiles) return;
-  const int warp = warp_id(), lane = lane_id();
+  const int warp = warp_uniform_id(), lane = lane_id();
   volatile int* abort_flag = &sm.abort_flag;
 
   if (threadIdx.x == 0) {
@@ -84,62 +84,71 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = sm.tmem_base;
+  const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
 
   if (warp == 0) {
-    if (lane == 0) {
-      uint32_t lc = 0;
-      bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        const int mt = t / n_tiles, nt = t - mt * n_tiles;
-        for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
-          const int st = lc % kStages;
-          ok = mbar_wait(&sm.empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
-          if (!ok) break;
+    // TMA producer: converged warp (warp-uniform coordinates), one elected lane issues.
+    uint32_t lc = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      const int mt = t / n_tiles, nt = t - mt * n_tiles;
+      for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
+        const int st = lc % kStages;
+        ok = mbar_wait_warp(&sm.empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
+        if (!ok) break;
+        if (elect_one()) {
           mbar_arrive_expect_tx(&sm.full[st], kABytes + kBBytes);
           tma_load_2d(sm.a[st], &tmap_a, &sm.full[st], kb * kBK, mt * kBM);
           tma_load_2d(sm.b[st], &tmap_b, &sm.full[st], kb * kBK, nt * kBN);
         }
+        __syncwarp();
       }
-      if (!ok) {
-        for (int s = 0; s < kStages; ++s) {
-          if (lc > (uint32_t)s) {
-            const uint32_t last = (lc - 1 - s) / kStages * kStages + s;
-            for (int i = 0; i < 1000000 && !mbar_try_wait(&sm.full[s], (last / kStages) & 1); ++i) {}
-          }
+    }
+    if (!ok && lane == 0) {
+      for (int s = 0; s < kStages; ++s) {
+        if (lc > (uint32_t)s) {
+          const uint32_t last = (lc - 1 - s) / kStages * kStages + s;
+          for (int i = 0; i < 1000000 && !mbar_try_wait(&sm.full[s], (last / kStages) & 1); ++i) {}
         }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(kBM, kBN, 0, 0);
-      uint32_t lc = 0, i = 0;
-      bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
-        const uint32_t ab = i & 1;
-        ok = mbar_wait(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1, prm.err, abort_flag);
+    // MMA issuer: converged warp; the elected lane (always the lowest, so the same one)
+    // issues the MMAs and the commits that track them.
+    const uint32_t idesc = idesc_bf16(kBM, kBN, 0, 0);
+    uint32_t lc = 0, i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++i) {
+      const uint32_t ab = i & 1;
+      ok = mbar_wait_warp(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1, prm.err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t d = tmem + ab * kBN;
+      for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
+        const int st = lc % kStages;
+        ok = mbar_wait_warp(&sm.full[st], (lc / kStages) & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t d = tmem + ab * kBN;
-        for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
-          const int st = lc % kStages;
-          ok = mbar_wait(&sm.full[st], (lc / kStages) & 1, prm.err, abort_flag);
-          if (!ok) break;
-          tc_fence_after();
-          const uint64_t da = sdesc_sw128(smem_u32(sm.a[st]));
-          const uint64_t db = sdesc_sw128(smem_u32(sm.b[st]));
+        const uint64_t da = sdesc_sw128(smem_u32(sm.a[st]));
+        const uint64_t db = sdesc_sw128(smem_u32(sm.b[st]));
+        if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
             tc_mma_ss(d, da + 2 * kk, db + 2 * kk, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
           tc_commit(&sm.empty[st]);
         }
-        if (!ok) break;
-        tc_commit(&sm.acc_full[ab]);
+        __syncwarp();
       }
-      if (!ok) {
+      if (!ok) break;
+      if (elect_one()) tc_commit(&sm.acc_full[ab]);
+      __syncwarp();
+    }
+    if (!ok) {
+      if (elect_one()) {
         tc_commit(&sm.drain);
         for (int it = 0; it < 1000000 && !mbar_try_wait(&sm.drain, 0); ++it) {}
       }
+      __syncwarp();
     }
   } else {
     const int e = warp - 2;                 // epilogue warp 0..7
@@ -151,8 +160,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
       const int mt = t / n_tiles, nt = t - mt * n_tiles;
       const uint32_t ab = i & 1;
-      bool ok = mbar_wait(&sm.acc_full[ab], (i >> 1) & 1, prm.err, abort_flag);
-      ok = __all_sync(0xffffffffu, ok);
+      const bool ok = mbar_wait_warp(&sm.acc_full[ab], (i >> 1) & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
       const int row0 = mt * kBM + quarter * 32;
@@ -214,7 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           // Stage the 32 x 32 block (row = lane, 64 bytes) in the 64-byte swizzle the
           // output tensor map uses: 16-byte chunk q of row r sits at chunk q ^ ((r >> 1) & 3).
           unsigned char* buf = stg + (nst & 1) * 2048;
-          if (lane == 0 && nst >= 2) tma_store_wait_read<1>();  // this buffer's last store read it
+          // The elected lane (lane 0, the lowest) owns this warp's bulk stores and their groups.
+          if (nst >= 2 && elect_one()) tma_store_wait_read<1>();  // this buffer's last store read it
           __syncwarp();
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
@@ -227,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) {
+          if (elect_one()) {
             tma_store_2d(&tmap_out, buf, col0, row0);
             tma_store_commit();
           }
@@ -240,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    if (lane == 0) tma_store_wait_all();
+    if (elect_one()) tma_store_wait_all();
     __syncwarp();
   }
 
