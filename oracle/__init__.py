@@ -16,7 +16,7 @@ textbook formulations without those storage roundings.  Mode decisions compare
 the saliency rounded to float32 with float32 thresholds, as the library does.
 
 Parity status: the router (§4.1), routing rule (§4.2), full and mean modes
-(Algorithm 1) and the block are pinned by tests in tests/test_oracle_*.py.  Two
+(Algorithm 1), the MaxAttn saliency (§3, appendix) and the block are pinned by tests in tests/test_oracle_*.py.  Two
 choices the paper leaves open are pinned only to the stated reading, not to a
 printed value: the scale of the routing attention (taken as beta_h / sqrt(d),
 beta_h = 1, like full attention) and the shape of MLP_gamma / MLP_delta
@@ -26,7 +26,8 @@ from .numerics import round_bf16, bf16_bits_to_f64, sigmoid, gelu, softmax, laye
 from .router import (pooling_logits, attention_pool, routing_vector, saliency,
                      select_mode, route_heads, bin_heads, MODE_MEAN, MODE_SURROGATE,
                      MODE_FULL, Q_TILE)
-from .modes import full_attention, surrogate_attention, mean_pooling, surrogate_mlp
+from .modes import (full_attention, surrogate_attention, mean_pooling, surrogate_mlp,
+                    max_attention_saliency)
 from .layer import (qkv_projection, head_router, moh_attention, global_block,
                     global_stack, load_layer)
 
@@ -35,6 +36,7 @@ __all__ = [
     "pooling_logits", "attention_pool", "routing_vector", "saliency", "select_mode",
     "route_heads", "bin_heads", "MODE_MEAN", "MODE_SURROGATE", "MODE_FULL", "Q_TILE",
     "full_attention", "surrogate_attention", "mean_pooling", "surrogate_mlp",
+    "max_attention_saliency",
     "qkv_projection", "head_router", "moh_attention", "global_block", "global_stack",
     "load_layer",
 ]

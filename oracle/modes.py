@@ -27,6 +27,21 @@ def full_attention(Q_h, K_h, V_h, rows=None, chunk=64):
     return out
 
 
+def max_attention_saliency(Q_h, K_h, chunk=64):
+    """MaxAttn saliency of a head (§3 "Head Saliency"; defined in the appendix section on
+    head saliency metrics): s_h^attn = max over all (i, j) of A_h[i, j], the largest entry
+    of the post-softmax attention matrix A_h = softmax(Q_h K_h^T / sqrt(d)).  Written out as
+    the definition: A_h row block by row block, then its maximum."""
+    Q_h = np.asarray(Q_h, np.float64)
+    K_h = np.asarray(K_h, np.float64)
+    d = Q_h.shape[1]
+    best = 0.0
+    for a in range(0, Q_h.shape[0], chunk):
+        A = softmax((Q_h[a:a + chunk] @ K_h.T) / np.sqrt(d), axis=1)
+        best = max(best, float(A.max()))
+    return best
+
+
 def surrogate_mlp(z, W1, b1, W2, b2):
     """MLP_gamma / MLP_delta of §4.3: Linear(2d -> L) -> GELU -> Linear(L -> d).
     The paper gives the hidden width (64, App. B) but not depth or activation;

@@ -125,3 +125,39 @@ def test_mean_pooling_closed_forms():
     yab, _ = oracle.mean_pooling(2 * A - 3 * B)
     np.testing.assert_allclose(yab, 2 * ya - 3 * yb, rtol=1e-12, atol=1e-13)
     np.testing.assert_allclose(ya[0], A.mean(0), rtol=1e-13)
+
+
+def test_max_attention_saliency_closed_forms():
+    """MaxAttn saliency s^attn = max_{i,j} A_ij (§3 and the appendix's saliency metrics)."""
+    g = np.random.default_rng(11)
+    N, d = 50, 64
+    # identical keys: every row of A is uniform, s = 1/N
+    K = np.tile(g.standard_normal(d), (N, 1))
+    assert abs(oracle.max_attention_saliency(g.standard_normal((7, d)), K) - 1.0 / N) < 1e-15
+    # one key scored gap g above the N-1 others for a single query: s = 1 / (1 + (N-1) e^-gap)
+    q = np.zeros((1, d)); q[0, 0] = 8.0  # scores = k[:, 0] (q.k / sqrt(64) = k0)
+    K = np.zeros((N, d)); K[3, 0] = 2.5
+    want = 1.0 / (1.0 + (N - 1) * np.exp(-2.5))
+    assert abs(oracle.max_attention_saliency(q, K) - want) < 1e-14
+    # several queries: the maximum over rows is taken (the peaked row wins over uniform ones)
+    Q = np.vstack([np.zeros((5, d)), q])
+    assert abs(oracle.max_attention_saliency(Q, K) - want) < 1e-14
+
+
+def test_max_attention_saliency_brute_force_and_invariances():
+    g = np.random.default_rng(12)
+    n, d = 9, 64
+    Q, K = 2 * g.standard_normal((n, d)), 2 * g.standard_normal((n + 4, d))
+    # brute force: each entry of A from its own numerator and denominator
+    best = 0.0
+    for i in range(n):
+        z = [float(np.dot(Q[i], K[j]) / 8.0) for j in range(n + 4)]
+        den = sum(np.exp(v) for v in z)
+        best = max(best, max(np.exp(v) / den for v in z))
+    s = oracle.max_attention_saliency(Q, K, chunk=4)
+    assert abs(s - best) < 1e-13
+    # invariant under permutations of queries and of keys; bounded by [1/N_k, 1]
+    assert abs(oracle.max_attention_saliency(Q[::-1], K[g.permutation(n + 4)]) - s) < 1e-13
+    assert 1.0 / (n + 4) <= s <= 1.0
+    # scaling the scores up sharpens A: s is non-decreasing in the score scale
+    assert oracle.max_attention_saliency(3 * Q, K) >= s
