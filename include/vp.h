@@ -167,11 +167,18 @@ vp_status vp_bin_heads(int32_t H, int32_t N, const int32_t* modes, int32_t* head
  *   surrogate heads: Y_h = C_h + sigma(MLP_gamma[v, C]) (.) MLP_delta[v, C]   (§4.3)
  *   mean heads:      Y_h = Broadcast(mean_v_h)
  *   y [N][H][d] bf16 (every head column is written).
+ *   s_attn [H] float or NULL: the MaxAttn saliency s_h^attn = max_{i,j} A_h[i, j] of every
+ *   full head (§3 "Head Saliency", defined in the appendix on saliency metrics: the largest
+ *   entry of the head's post-softmax attention matrix), computed exactly, as a by-product of
+ *   the flash kernel, from each query row's softmax denominator relative to its true maximum
+ *   (max_j A_ij = 1 / sum_j exp(S_ij - max_j S_ij)).  Heads not in full mode get 0 (their
+ *   attention matrix is never formed): force every head to full mode to obtain the exact
+ *   saliency of all heads, e.g. to compare it with the router's estimate s_h.
  */
 vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32_t* head_ids,
                             const int32_t* offsets, const float* ctx, const float* mean_v,
-                            const vp_surrogate_weights* sw, vp_bf16* y, void* ws, size_t ws_bytes,
-                            void* stream);
+                            const vp_surrogate_weights* sw, vp_bf16* y, float* s_attn, void* ws,
+                            size_t ws_bytes, void* stream);
 
 /*
  * vp_linear -- out = residual + scale (.) act(A W^T + bias), the dense projections of
@@ -197,26 +204,28 @@ vp_status vp_layer_norm(int32_t M, int32_t D, const vp_bf16* x, const float* gam
  * QKV = x W_qkv^T + b_qkv, router, bins and per-mode heads in between.
  *   x [N][D] bf16; out [N][D] bf16; force_modes [H] or NULL (see vp_router).
  *   qkv_out [N][3D] / y_out [N][D] bf16 or NULL: copies of the intermediates (debug).
- *   s_out [H] float / modes_out [H] int32 or NULL.
+ *   s_out [H] float / modes_out [H] int32 or NULL; s_attn_out [H] float or NULL: MaxAttn
+ *   saliency of the full heads (see vp_head_attention).
  */
 vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const vp_bf16* w_qkv,
                                   const float* b_qkv, const vp_bf16* w_o, const float* b_o,
                                   const vp_router_weights* rw, const vp_surrogate_weights* sw,
                                   const int32_t* force_modes, vp_bf16* out, vp_bf16* qkv_out,
-                                  vp_bf16* y_out, float* s_out, int32_t* modes_out, void* ws,
-                                  size_t ws_bytes, void* stream);
+                                  vp_bf16* y_out, float* s_out, float* s_attn_out,
+                                  int32_t* modes_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * vp_global_stack -- n_layers global blocks (Algorithm 1) applied in place to x_inout
  * [N][D] bf16.  layers: HOST array of n_layers vp_layer_weights (their tensors are device
- * pointers).  force_modes [n_layers][H] int32 or NULL; modes_out / s_out [n_layers][H] or
- * NULL.  ln_eps: LayerNorm epsilon (the paper does not state it; 1e-6 in the tests).
+ * pointers).  force_modes [n_layers][H] int32 or NULL; modes_out / s_out / s_attn_out
+ * [n_layers][H] or NULL (s_attn_out: MaxAttn saliency of the full heads, see
+ * vp_head_attention).  ln_eps: LayerNorm epsilon (the paper does not state it; 1e-6 in the tests).
  * Every weight, bias, LayerNorm and LayerScale pointer must be 16-byte aligned.
  */
 vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
                           const vp_layer_weights* layers, const int32_t* force_modes,
-                          int32_t* modes_out, float* s_out, float ln_eps, void* ws,
-                          size_t ws_bytes, void* stream);
+                          int32_t* modes_out, float* s_out, float* s_attn_out, float ln_eps,
+                          void* ws, size_t ws_bytes, void* stream);
 
 /*
  * vp_router_noalloc -- vp_router without a workspace, for callers that cannot allocate

@@ -120,7 +120,7 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
     F = (Hd @ lw["w_fc2"].T + lw["b_fc2"]) * lw["ls2"]
     X_next = mat(X_attn + F)
     return X_next, {"modes": att["modes"], "natural_modes": att["natural_modes"],
-                    "s": att["s"], "X_attn": X_attn}
+                    "s": att["s"], "X_attn": X_attn, "qkv": att["qkv"]}
 
 
 def global_stack(X, layers, force_modes=None, materialize=round_bf16, eps=LN_EPS):

@@ -69,7 +69,8 @@ _SIGS = [
     ("vp_bin_heads", c_int32, [c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                c_void_p]),
     ("vp_head_attention", c_int32, [POINTER(VpDims), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
-                                    POINTER(VpSurrogateWeights), c_void_p, c_void_p, c_size_t, c_void_p]),
+                                    POINTER(VpSurrogateWeights), c_void_p, c_void_p, c_void_p, c_size_t,
+                                    c_void_p]),
     ("vp_linear", c_int32, [c_int32, c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_int32, c_void_p,
                             c_void_p, c_void_p, c_void_p]),
     ("vp_layer_norm", c_int32, [c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_float, c_void_p,
@@ -77,11 +78,13 @@ _SIGS = [
     ("vp_moh_global_attention", c_int32, [POINTER(VpDims), c_void_p, c_void_p, c_void_p, c_void_p,
                                           c_void_p, POINTER(VpRouterWeights),
                                           POINTER(VpSurrogateWeights), c_void_p, c_void_p, c_void_p,
-                                          c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+                                          c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
+                                          c_void_p]),
     ("vp_profile_begin", c_int32, [c_int32]),
     ("vp_profile_end", c_int32, [POINTER(c_int32), POINTER(c_int32), POINTER(c_float)]),
     ("vp_global_stack", c_int32, [POINTER(VpDims), c_int32, c_void_p, POINTER(VpLayerWeights),
-                                  c_void_p, c_void_p, c_void_p, c_float, c_void_p, c_size_t, c_void_p]),
+                                  c_void_p, c_void_p, c_void_p, c_void_p, c_float, c_void_p, c_size_t,
+                                  c_void_p]),
 ]
 EXPORTS = [s[0] for s in _SIGS]
 
@@ -208,9 +211,10 @@ def vp_bin_heads(H, N, modes, head_ids, offsets, work=None, n_work=None, stream=
                               _stream(stream)), "vp_bin_heads")
 
 
-def vp_head_attention(dm, qkv, head_ids, offsets, ctx, mean_v, sw: VpSurrogateWeights, y, ws, stream=None):
+def vp_head_attention(dm, qkv, head_ids, offsets, ctx, mean_v, sw: VpSurrogateWeights, y, ws, stream=None,
+                      s_attn=None):
     _check(lib().vp_head_attention(ctypes.byref(dm), _p(qkv), _p(head_ids), _p(offsets), _p(ctx), _p(mean_v),
-                                   ctypes.byref(sw), _p(y), _p(ws), ws.numel(), _stream(stream)),
+                                   ctypes.byref(sw), _p(y), _p(s_attn), _p(ws), ws.numel(), _stream(stream)),
            "vp_head_attention")
 
 
@@ -234,17 +238,18 @@ def vp_layer_norm(x, gamma, beta, eps=1e-6, out=None, stream=None):
 
 
 def vp_moh_global_attention(dm, x, w_qkv, b_qkv, w_o, b_o, rw, sw, force_modes, out, qkv_out, y_out,
-                            s_out, modes_out, ws, stream=None):
+                            s_out, modes_out, ws, stream=None, s_attn_out=None):
     _check(lib().vp_moh_global_attention(ctypes.byref(dm), _p(x), _p(w_qkv), _p(b_qkv), _p(w_o), _p(b_o),
                                          ctypes.byref(rw), ctypes.byref(sw), _p(force_modes), _p(out),
-                                         _p(qkv_out), _p(y_out), _p(s_out), _p(modes_out), _p(ws),
-                                         ws.numel(), _stream(stream)), "vp_moh_global_attention")
+                                         _p(qkv_out), _p(y_out), _p(s_out), _p(s_attn_out), _p(modes_out),
+                                         _p(ws), ws.numel(), _stream(stream)), "vp_moh_global_attention")
 
 
-def vp_global_stack(dm, x_inout, layers, force_modes, modes_out, s_out, ln_eps, ws, stream=None):
+def vp_global_stack(dm, x_inout, layers, force_modes, modes_out, s_out, ln_eps, ws, stream=None,
+                    s_attn_out=None):
     arr = (VpLayerWeights * len(layers))(*layers)
     _check(lib().vp_global_stack(ctypes.byref(dm), len(layers), _p(x_inout), arr, _p(force_modes),
-                                 _p(modes_out), _p(s_out), float(ln_eps), _p(ws), ws.numel(),
+                                 _p(modes_out), _p(s_out), _p(s_attn_out), float(ln_eps), _p(ws), ws.numel(),
                                  _stream(stream)), "vp_global_stack")
 
 

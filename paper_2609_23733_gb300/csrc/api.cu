@@ -216,8 +216,8 @@ SurrogateArgs make_surrogate_args(const vp_surrogate_weights* sw) {
 // Runs the three mode kernels for bins already in device memory.
 vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* head_ids,
                     const int32_t* offsets, const float* ctx, const float* mean_v,
-                    const vp_surrogate_weights* sw, __nv_bfloat16* y, const RouterScratch& sc,
-                    cudaStream_t st) {
+                    const vp_surrogate_weights* sw, __nv_bfloat16* y, float* s_attn,
+                    const RouterScratch& sc, cudaStream_t st) {
   HeadAttnArgs ha{};
   ha.N = dm->N;
   ha.H = dm->H;
@@ -228,6 +228,7 @@ vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* 
   ha.mean_v = mean_v;
   ha.sw = make_surrogate_args(sw);
   ha.y = y;
+  ha.s_attn = s_attn;
   ha.err = sc.err;
   ha.cheap_counter = sc.cheap_counter;
   return from_cuda(launch_heads(ha, device_sm_count(), st));
@@ -239,7 +240,8 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
                     const __nv_bfloat16* residual, const vp_router_weights* rw,
                     const vp_surrogate_weights* sw, const int32_t* force_modes,
                     __nv_bfloat16* out, __nv_bfloat16* qkv, __nv_bfloat16* y, float* s_out,
-                    int32_t* modes_out, const RouterScratch& sc, cudaStream_t st) {
+                    float* s_attn_out, int32_t* modes_out, const RouterScratch& sc,
+                    cudaStream_t st) {
   const int N = dm->N, D = dm->H * kHeadDim;
   const int sms = device_sm_count();
   LinearArgs la{};
@@ -257,7 +259,8 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
   ra.s_out = s_out;
   ra.modes_out = modes_out;
   VP_TRY(from_cuda(launch_router(ra, sc, sms, st)));
-  VP_TRY(run_heads(dm, qkv, sc.head_ids, sc.offsets, sc.ctx, sc.mean_v, sw, y, sc, st));
+  VP_TRY(run_heads(dm, qkv, sc.head_ids, sc.offsets, sc.ctx, sc.mean_v, sw, y, s_attn_out, sc,
+                   st));
   LinearArgs lo{};
   lo.M = N;
   lo.N = D;
@@ -398,8 +401,8 @@ vp_status vp_bin_heads(int32_t H, int32_t N, const int32_t* modes, int32_t* head
 
 vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32_t* head_ids,
                             const int32_t* offsets, const float* ctx, const float* mean_v,
-                            const vp_surrogate_weights* sw, vp_bf16* y, void* ws, size_t ws_bytes,
-                            void* stream) {
+                            const vp_surrogate_weights* sw, vp_bf16* y, float* s_attn, void* ws,
+                            size_t ws_bytes, void* stream) {
   VP_TRY(check_dims(dims));
   if (!qkv || !head_ids || !offsets || !ctx || !mean_v || !y) return VP_ERR_INVALID_ARG;
   if (!aligned16(qkv) || !aligned16(y)) return VP_ERR_ALIGNMENT;
@@ -408,7 +411,7 @@ vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32
   VP_TRY(check_device());
   RouterScratch sc = carve_router_scratch(ws, dims->H);
   return run_heads(dims, reinterpret_cast<const __nv_bfloat16*>(qkv), head_ids, offsets, ctx,
-                   mean_v, sw, reinterpret_cast<__nv_bfloat16*>(y), sc,
+                   mean_v, sw, reinterpret_cast<__nv_bfloat16*>(y), s_attn, sc,
                    static_cast<cudaStream_t>(stream));
 }
 
@@ -456,8 +459,8 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
                                   const float* b_qkv, const vp_bf16* w_o, const float* b_o,
                                   const vp_router_weights* rw, const vp_surrogate_weights* sw,
                                   const int32_t* force_modes, vp_bf16* out, vp_bf16* qkv_out,
-                                  vp_bf16* y_out, float* s_out, int32_t* modes_out, void* ws,
-                                  size_t ws_bytes, void* stream) {
+                                  vp_bf16* y_out, float* s_out, float* s_attn_out,
+                                  int32_t* modes_out, void* ws, size_t ws_bytes, void* stream) {
   VP_TRY(check_dims(dims));
   if (!x || !w_qkv || !w_o || !out) return VP_ERR_INVALID_ARG;
   if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(w_o) || !aligned16(out) ||
@@ -479,13 +482,13 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
   if (y_out) y = reinterpret_cast<__nv_bfloat16*>(y_out);
   return run_layer(dims, reinterpret_cast<const __nv_bfloat16*>(x), w_qkv, b_qkv, w_o, b_o,
                    nullptr, nullptr, rw, sw, force_modes, reinterpret_cast<__nv_bfloat16*>(out),
-                   qkv, y, s_out, modes_out, sc, st);
+                   qkv, y, s_out, s_attn_out, modes_out, sc, st);
 }
 
 vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
                           const vp_layer_weights* layers, const int32_t* force_modes,
-                          int32_t* modes_out, float* s_out, float ln_eps, void* ws,
-                          size_t ws_bytes, void* stream) {
+                          int32_t* modes_out, float* s_out, float* s_attn_out, float ln_eps,
+                          void* ws, size_t ws_bytes, void* stream) {
   VP_TRY(check_dims(dims));
   if (n_layers < 1 || !x_inout || !layers) return VP_ERR_INVALID_ARG;
   if (!aligned16(x_inout)) return VP_ERR_ALIGNMENT;
@@ -526,6 +529,7 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     VP_TRY(run_layer(dims, xt, w.w_qkv, w.b_qkv, w.w_o, w.b_o, w.ls1, x, &w.router, &w.surrogate,
                      force_modes ? force_modes + (size_t)l * dims->H : nullptr, x, qkv, y,
                      s_out ? s_out + (size_t)l * dims->H : nullptr,
+                     s_attn_out ? s_attn_out + (size_t)l * dims->H : nullptr,
                      modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st));
     // (4) Z~ = LN2(X_attn); X <- X_attn + LS2 FFN(Z~)
     VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, xt, st)));

@@ -18,6 +18,7 @@
 // products, and S_c(j+1) is issued as soon as chain c has read S_c(j).
 // TMEM: S_0 [0,128) S_1 [128,256) O_0 [256,320) O_1 [320,384) P_0 [384,448) P_1 [448,512).
 // Keys past N are zero-filled by TMA and masked to -inf; query rows past N are not stored.
+// Optionally the epilogue also yields the head's MaxAttn saliency max_ij A_ij (§3).
 // Every CTA signals its dependents at once (griddepcontrol.launch_dependents), so the
 // cheap-heads kernel queued behind this one (heads_cheap.cu) can take the SMs that the last
 // full-attention round leaves idle.
@@ -57,6 +58,7 @@ struct FullParams {
   const int32_t* head_ids;
   const int32_t* offsets;
   __nv_bfloat16* y;
+  float* s_attn;  // [H] MaxAttn saliency (zeroed by the launcher), or NULL
   unsigned int* err;
 };
 
@@ -246,7 +248,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int item = blockIdx.x; item < items && ok; item += gridDim.x) {
       const int h = __ldg(prm.head_ids + first + item / n_pairs);
       const int qp = item % n_pairs;
-      float m = 0.f, lsum = 0.f;
+      // m: the (lazily updated) reference the exponentials are taken against; xmax: the
+      // true running maximum of the row's scaled scores, for the MaxAttn saliency.
+      float m = 0.f, lsum = 0.f, xmax = 0.f;
       for (int j = 0; j < n_kv; ++j, ++g) {
         ok = mbar_wait_warp(&sm.s_full[c], g & 1, prm.err, abort_flag);
         if (!ok) break;
@@ -277,6 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mx = fmaxf(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], fmax3(t[5], t[6], t[7])));
         }
         const float mx2 = mx * cs;
+        xmax = j == 0 ? mx2 : fmaxf(xmax, mx2);
         float alpha = 1.f;
         bool need = false;
         if (j == 0) {
@@ -338,8 +343,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive(&sm.o_empty[c]);
       const int row = qp * 2 * kBM + c * kBM + row_in_tile;
+      const float inv = 1.f / lsum;
       if (row < N) {
-        const float inv = 1.f / lsum;
         uint4* dst = reinterpret_cast<uint4*>(prm.y + ((size_t)row * H + h) * 64);
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {
@@ -350,6 +355,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           v.w = pack_bf16x2(o[8 * ch + 6] * inv, o[8 * ch + 7] * inv);
           dst[ch] = v;
         }
+      }
+      if (prm.s_attn) {
+        // MaxAttn saliency (§3): the largest entry of row i of A is 2^(xmax - m) / lsum (the
+        // row's maximum over its softmax denominator); the head's value is the maximum over
+        // rows, folded in with an integer atomic max (the values are positive floats).
+        float a = row < N ? fast_exp2(xmax - m) * inv : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+        if (lane == 0) atomicMax(reinterpret_cast<int*>(prm.s_attn + h), __float_as_int(a));
       }
       __syncwarp();
     }
@@ -373,7 +387,7 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
   const int smem = (int)sizeof(FullSmem) + 1024;
   e = cudaFuncSetAttribute(attn_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.err};
+  FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.s_attn, a.err};
   attn_full_kernel<<<num_sms, kThreads, smem, st>>>(tmap, prm);
   return cudaGetLastError();
 }

@@ -81,6 +81,7 @@ struct HeadAttnArgs {
   const float* mean_v;
   SurrogateArgs sw;
   __nv_bfloat16* y;
+  float* s_attn;                // [H] MaxAttn saliency of the full heads, or NULL
   unsigned int* err;
   unsigned int* cheap_counter;  // one word of scratch, zeroed by the launcher
 };

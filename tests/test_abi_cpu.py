@@ -91,7 +91,8 @@ def test_host_side_validation(vp):
     # vp_bin_heads: no heads
     assert lib.vp_bin_heads(0, 10, A, A, A, None, None, None) == 2
     # vp_global_stack: no layers
-    assert lib.vp_global_stack(ctypes.byref(dm), 0, A, None, None, None, None, ctypes.c_float(1e-6), A, 1 << 30, None) == 1
+    assert lib.vp_global_stack(ctypes.byref(dm), 0, A, None, None, None, None, None, ctypes.c_float(1e-6), A,
+                               1 << 30, None) == 1
 
 
 def test_valid_call_without_a_gpu_reports_the_device(vp):

@@ -202,20 +202,34 @@ def test_bin_heads_bit_exact():
 
 
 # ------------------------------------------------------------------ head modes (a6, a7, a8)
-def _run_heads(qkv_bits, w, N, H, modes, ctx, mean_v):
+def _run_heads(qkv_bits, w, N, H, modes, ctx, mean_v, with_saliency=False):
     dm = vpb.dims(N, H)
     dw = vpb.to_device(w)
     sw = vpb.surrogate_weights(dw)
     ws = vpb.workspace(dm, vpb.VP_WS_ROUTER)
     ids_o, off_o, _ = oracle.bin_heads(modes, N)
     y = torch.full((N, H * 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+    s_attn = torch.full((H,), float("nan"), device="cuda") if with_saliency else None
     vpb.vp_head_attention(dm, vpb.bf16_from_bits(qkv_bits.reshape(N, -1)),
                           torch.tensor(ids_o, device="cuda"), torch.tensor(off_o, device="cuda"),
                           torch.tensor(ctx, dtype=torch.float32, device="cuda"),
-                          torch.tensor(mean_v, dtype=torch.float32, device="cuda"), sw, y, ws)
+                          torch.tensor(mean_v, dtype=torch.float32, device="cuda"), sw, y, ws,
+                          s_attn=s_attn)
     torch.cuda.synchronize()
     assert vpb.vp_read_device_error(ws) == 0
-    return _f64(y).reshape(N, H, 64)
+    out = _f64(y).reshape(N, H, 64)
+    return (out, s_attn.cpu().numpy().astype(np.float64)) if with_saliency else out
+
+
+def _check_saliency(s_attn, qkv, modes, what):
+    """MaxAttn saliency of the full heads against the oracle's definition (same bf16 Q, K;
+    the kernel's fp32 scores, sums and exponentials leave ~1e-5 relative); 0 elsewhere."""
+    for h in range(len(modes)):
+        if modes[h] == 2:
+            want = oracle.max_attention_saliency(qkv[:, 0, h], qkv[:, 1, h])
+            assert abs(s_attn[h] - want) <= 1e-3 * want, (what, h, s_attn[h], want)
+        else:
+            assert s_attn[h] == 0.0, (what, h, s_attn[h])
 
 
 @pytest.mark.parametrize("N", [1, 5, 127, 128, 129, 300, 1044, 2000])
@@ -241,9 +255,10 @@ def test_head_modes_match_oracle(N):
             want[:, h], _ = oracle.surrogate_attention(V, r, mg, md)
         else:
             want[:, h], _ = oracle.mean_pooling(V)
-    got = _run_heads(qkv_bits, w, N, H, modes, ctx, mean_v)
+    got, s_attn = _run_heads(qkv_bits, w, N, H, modes, ctx, mean_v, with_saliency=True)
     for h in range(H):
         compare(got[:, h], oracle.round_bf16(want[:, h]), what=f"head {h} mode {modes[h]}")
+    _check_saliency(s_attn, qkv, modes, f"N={N}")
 
 
 @pytest.mark.parametrize("N", [5000, 9999])
@@ -274,10 +289,34 @@ def test_full_attention_peaked_scores():
     qkv_bits = synth.f32_to_bf16_bits(qkv)
     w = synth.make_layer_weights(synth.rng(0), D=H * 64, H=H)
     q = oracle.bf16_bits_to_f64(qkv_bits).reshape(N, 3, H, 64)
-    got = _run_heads(qkv_bits, w, N, H, np.array([2, 2], np.int32), np.zeros((H, 64)), np.zeros((H, 64)))
+    got, s_attn = _run_heads(qkv_bits, w, N, H, np.array([2, 2], np.int32), np.zeros((H, 64)),
+                             np.zeros((H, 64)), with_saliency=True)
     for h in range(H):
         compare(got[:, h], oracle.round_bf16(oracle.full_attention(q[:, 0, h], q[:, 1, h], q[:, 2, h])),
                 what=f"peaked head {h}")
+    # the row maxima move after the first key tiles here, so the saliency needs the true row
+    # maximum, not the lazily updated reference of the exponentials
+    _check_saliency(s_attn, q, [2, 2], "peaked")
+
+
+def test_max_attention_saliency_closed_forms():
+    """Identical keys: every entry of A is 1/N.  One key scored g above the others for every
+    query: s = 1 / (1 + (N - 1) e^-g).  Both at sizes spanning several key tiles."""
+    H, N = 2, 1000
+    g = np.random.default_rng(21)
+    qkv = np.zeros((N, 3, H, 64), np.float32)
+    qkv[:, 0] = g.standard_normal((N, H, 64))
+    qkv[:, 1, 0] = g.standard_normal(64)          # head 0: identical keys
+    qkv[:, 0, 1] = 0.0
+    qkv[:, 0, 1, 0] = 8.0                         # head 1: score = k_j[0]
+    qkv[777, 1, 1, 0] = 2.5                       # one key 2.5 above the rest (0)
+    qkv[:, 2] = g.standard_normal((N, H, 64))
+    w = synth.make_layer_weights(synth.rng(0), D=H * 64, H=H)
+    _, s_attn = _run_heads(synth.f32_to_bf16_bits(qkv), w, N, H, np.array([2, 2], np.int32),
+                           np.zeros((H, 64)), np.zeros((H, 64)), with_saliency=True)
+    assert abs(s_attn[0] - 1.0 / N) <= 1e-5 / N
+    want = 1.0 / (1.0 + (N - 1) * np.exp(-2.5))
+    assert abs(s_attn[1] - want) <= 1e-5 * want
 
 
 # ------------------------------------------------------------------ whole layer
@@ -288,13 +327,15 @@ def _run_layer(x_bits, w, N, H, force=None):
     D = H * 64
     out = torch.zeros(N, D, dtype=torch.bfloat16, device="cuda")
     s = torch.zeros(H, device="cuda")
+    s_attn = torch.full((H,), float("nan"), device="cuda")
     modes = torch.zeros(H, dtype=torch.int32, device="cuda")
     fm = None if force is None else torch.tensor(force, dtype=torch.int32, device="cuda")
     vpb.vp_moh_global_attention(dm, vpb.bf16_from_bits(x_bits), dw["w_qkv"], dw["b_qkv"], dw["w_o"],
                                 dw["b_o"], vpb.router_weights(dw), vpb.surrogate_weights(dw), fm, out,
-                                None, None, s, modes, ws)
+                                None, None, s, modes, ws, s_attn_out=s_attn)
     torch.cuda.synchronize()
     assert vpb.vp_read_device_error(ws) == 0
+    _run_layer.s_attn = s_attn.cpu().numpy().astype(np.float64)
     return _f64(out), s.cpu().numpy(), modes.cpu().numpy()
 
 
@@ -310,6 +351,14 @@ def test_layer_s4_224(force):
     compare(got, want["out"], what="layer out")
     np.testing.assert_allclose(s, want["s"], rtol=2e-3)
     np.testing.assert_array_equal(modes, want["modes"])
+    # MaxAttn saliency of the full heads; both sides round their own QKV to bf16, which moves
+    # a score by ~1e-3 at most
+    for h in range(16):
+        if modes[h] == synth.MODE_FULL:
+            ref = oracle.max_attention_saliency(want["qkv"][:, 0, h], want["qkv"][:, 1, h])
+            assert abs(_run_layer.s_attn[h] - ref) <= 1e-2 * ref, (h, _run_layer.s_attn[h], ref)
+        else:
+            assert _run_layer.s_attn[h] == 0.0
     if force is None:
         # Untrained routers: every head is diffuse, saliency ~ 1/N, so every head is mean.
         assert np.all(want["natural_modes"] == synth.MODE_MEAN)

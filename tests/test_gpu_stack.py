@@ -38,10 +38,12 @@ def _run_stack(x_bits, ws_host, N, force=None, H=16):
     L = len(ws_host)
     modes = torch.full((L, H), -1, dtype=torch.int32, device="cuda")
     s = torch.zeros(L, H, device="cuda")
+    s_attn = torch.full((L, H), float("nan"), device="cuda")
     fm = None if force is None else torch.tensor(np.asarray(force, np.int32), device="cuda")
-    vpb.vp_global_stack(dm, x, layers, fm, modes, s, 1e-6, ws)
+    vpb.vp_global_stack(dm, x, layers, fm, modes, s, 1e-6, ws, s_attn_out=s_attn)
     torch.cuda.synchronize()
     assert vpb.vp_read_device_error(ws) == 0
+    _run_stack.s_attn = s_attn.cpu().numpy().astype(np.float64)
     return _f64(x), modes.cpu().numpy(), s.cpu().numpy()
 
 
@@ -60,6 +62,17 @@ def test_stack_three_blocks_all_modes():
     np.testing.assert_array_equal(modes, force)
     np.testing.assert_allclose(s[0], infos[0]["s"], rtol=5e-3)
     compare(got, want, rel=L * BF16_STEP, what="3-block stack")
+    # MaxAttn saliency per block for the full heads (0 for the others); later blocks see the
+    # residual stream after the earlier blocks' independent roundings, hence 2 %
+    for l in range(L):
+        for h in range(16):
+            got_s = _run_stack.s_attn[l, h]
+            if force[l][h] == synth.MODE_FULL:
+                q = infos[l]["qkv"]
+                ref = oracle.max_attention_saliency(q[:, 0, h], q[:, 1, h])
+                assert abs(got_s - ref) <= 2e-2 * ref, (l, h, got_s, ref)
+            else:
+                assert got_s == 0.0, (l, h, got_s)
 
 
 def test_stack_24_blocks_s4_natural_routing():
