@@ -27,16 +27,16 @@ from .router import (pooling_logits, attention_pool, routing_vector, saliency,
                      select_mode, route_heads, bin_heads, MODE_MEAN, MODE_SURROGATE,
                      MODE_FULL, Q_TILE)
 from .modes import (full_attention, surrogate_attention, mean_pooling, surrogate_mlp,
-                    max_attention_saliency)
+                    max_attention_saliency, elu_feature_map, linear_attention)
 from .layer import (qkv_projection, head_router, moh_attention, global_block,
-                    global_stack, load_layer)
+                    global_stack, load_layer, VARIANTS)
 
 __all__ = [
     "round_bf16", "bf16_bits_to_f64", "sigmoid", "gelu", "softmax", "layer_norm",
     "pooling_logits", "attention_pool", "routing_vector", "saliency", "select_mode",
     "route_heads", "bin_heads", "MODE_MEAN", "MODE_SURROGATE", "MODE_FULL", "Q_TILE",
     "full_attention", "surrogate_attention", "mean_pooling", "surrogate_mlp",
-    "max_attention_saliency",
+    "max_attention_saliency", "elu_feature_map", "linear_attention", "VARIANTS",
     "qkv_projection", "head_router", "moh_attention", "global_block", "global_stack",
     "load_layer",
 ]

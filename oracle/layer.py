@@ -10,7 +10,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from .modes import full_attention, mean_pooling, surrogate_attention
+from .modes import full_attention, linear_attention, mean_pooling, surrogate_attention
 from .numerics import bf16_bits_to_f64, gelu, layer_norm, round_bf16
 from .router import MODE_FULL, MODE_SURROGATE, attention_pool, routing_vector, saliency, select_mode
 
@@ -44,26 +44,33 @@ def qkv_projection(Xt, lw, materialize=round_bf16):
     return qkv.reshape(N, 3, H, -1)
 
 
-def head_router(Q_h, K_h, lw, h, beta=None):
+# Ablation variants of §5 (component ablation and compute-mode ablation).  Two-branch
+# routing (mean and full only) is tau_low == tau_high with the ordinary routing rule.
+VARIANTS = ("mean_qpool", "mean_context", "no_residual", "linear_attention")
+
+
+def head_router(Q_h, K_h, lw, h, beta=None, mean_qpool=False):
     """§4.1 for head h: (alpha, q_pool, r_h, s_h)."""
     d = Q_h.shape[1]
     alpha, q_pool = attention_pool(Q_h, lw["r_W"][h], lw["r_U"][h], lw["r_w"][h],
-                                   lw["r_bW"][h], lw["r_bU"][h])
+                                   lw["r_bW"][h], lw["r_bU"][h], mean_pool=mean_qpool)
     b = lw["r_beta"][h] if beta is None else beta
     r = routing_vector(q_pool, K_h, b / np.sqrt(d))
     return alpha, q_pool, r, saliency(r)
 
 
 def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
-                  tau_low=TAU_LOW, tau_high=TAU_HIGH):
+                  tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=()):
     """Routed multi-head attention of one layer (Algorithm 1 steps 2-3 up to W_O).
 
     X [N, D] float64 (the block passes LN1(X)); lw from load_layer.
     force_modes [H] replaces the routing decision only (the router still runs;
     surrogate heads still use its r_h).  ``rows`` restricts the per-token
     outputs to a subset of query rows (all rows when None); router statistics
-    always use every token.
+    always use every token.  ``variant``: names from VARIANTS (§5 ablations).
     """
+    variant = set(variant)
+    assert variant <= set(VARIANTS), variant
     mat = materialize or _identity
     X = np.asarray(X, np.float64)
     N = X.shape[0]
@@ -77,7 +84,7 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
     modes = np.zeros(H, np.int32)
     for h in range(H):
         Q_h, K_h, V_h = qkv[:, 0, h], qkv[:, 1, h], qkv[:, 2, h]
-        alpha, q_pool, r, s = head_router(Q_h, K_h, lw, h)
+        alpha, q_pool, r, s = head_router(Q_h, K_h, lw, h, mean_qpool="mean_qpool" in variant)
         res["alpha"].append(alpha)
         res["r"].append(r)
         res["q_pool"][h] = q_pool
@@ -88,10 +95,14 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
         res["mean_v"][h] = V_h.sum(axis=0) / N
         if modes[h] == MODE_FULL:
             Y[:, h] = full_attention(Q_h, K_h, V_h, rows=idx)
+        elif modes[h] == MODE_SURROGATE and "linear_attention" in variant:
+            Y[:, h] = linear_attention(Q_h, K_h, V_h, rows=idx)
         elif modes[h] == MODE_SURROGATE:
             mg = (lw["s_g1_w"][h], lw["s_g1_b"][h], lw["s_g2_w"][h], lw["s_g2_b"][h])
             md = (lw["s_d1_w"][h], lw["s_d1_b"][h], lw["s_d2_w"][h], lw["s_d2_b"][h])
-            Y[:, h], _ = surrogate_attention(V_h, r, mg, md, rows=idx)
+            Y[:, h], _ = surrogate_attention(V_h, r, mg, md, rows=idx,
+                                             mean_context="mean_context" in variant,
+                                             residual="no_residual" not in variant)
         else:
             Y[:, h], _ = mean_pooling(V_h, n_rows=len(idx))
     res["natural_modes"] = natural
@@ -102,7 +113,7 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
 
 
 def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
-                 tau_low=TAU_LOW, tau_high=TAU_HIGH):
+                 tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=()):
     """Algorithm 1 (VGGT-Prime global aggregator block), all rows.
 
     (1) X~ = LN1(X); (2) routed attention -> Y; (3) A = LS1(Y W_O),
@@ -112,7 +123,7 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
     X = np.asarray(X, np.float64)
     Xt = mat(layer_norm(X, lw["ln1_g"], lw["ln1_b"], eps))
     att = moh_attention(Xt, lw, force_modes=force_modes, materialize=materialize,
-                        tau_low=tau_low, tau_high=tau_high)
+                        tau_low=tau_low, tau_high=tau_high, variant=variant)
     A = (att["Y"] @ lw["w_o"].T + lw["b_o"]) * lw["ls1"]
     X_attn = mat(X + A)
     Zt = mat(layer_norm(X_attn, lw["ln2_g"], lw["ln2_b"], eps))
@@ -123,12 +134,13 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
                     "s": att["s"], "X_attn": X_attn, "qkv": att["qkv"]}
 
 
-def global_stack(X, layers, force_modes=None, materialize=round_bf16, eps=LN_EPS):
+def global_stack(X, layers, force_modes=None, materialize=round_bf16, eps=LN_EPS, variant=()):
     """Algorithm 1 applied layer after layer.  force_modes: [n_layers, H] or None.
     Returns (X_out, list of per-layer info)."""
     infos = []
     for l, lw in enumerate(layers):
         fm = None if force_modes is None else force_modes[l]
-        X, info = global_block(X, lw, force_modes=fm, materialize=materialize, eps=eps)
+        X, info = global_block(X, lw, force_modes=fm, materialize=materialize, eps=eps,
+                               variant=variant)
         infos.append(info)
     return X, infos

@@ -31,10 +31,17 @@ def pooling_logits(Q_h, W_h, U_h, w_h, bW=None, bU=None):
     return (np.tanh(a) * sigmoid(b)) @ np.asarray(w_h, np.float64)
 
 
-def attention_pool(Q_h, W_h, U_h, w_h, bW=None, bU=None):
+def attention_pool(Q_h, W_h, U_h, w_h, bW=None, bU=None, mean_pool=False):
     """§4.1: alpha_h = softmax over all N tokens of the pooling logits;
-    q_pool = sum_i alpha_{h,i} q_{h,i}.  Returns (alpha [N], q_pool [d])."""
-    alpha = softmax(pooling_logits(Q_h, W_h, U_h, w_h, bW, bU))
+    q_pool = sum_i alpha_{h,i} q_{h,i}.  Returns (alpha [N], q_pool [d]).
+
+    mean_pool: the component ablation of §5 ("Q-Pooling" replaced by mean pooling):
+    alpha = 1/N for every token, q_pool = the mean query."""
+    if mean_pool:
+        N = np.asarray(Q_h).shape[0]
+        alpha = np.full(N, 1.0 / N)
+    else:
+        alpha = softmax(pooling_logits(Q_h, W_h, U_h, w_h, bW, bU))
     return alpha, alpha @ np.asarray(Q_h, np.float64)
 
 

@@ -161,3 +161,71 @@ def test_max_attention_saliency_brute_force_and_invariances():
     assert 1.0 / (n + 4) <= s <= 1.0
     # scaling the scores up sharpens A: s is non-decreasing in the score scale
     assert oracle.max_attention_saliency(3 * Q, K) >= s
+
+
+# ------------------------------------------------------------------ §5 ablation variants
+def _mlps(g, d=64, L=64, delta_zero=False):
+    def mlp(zero=False):
+        W1 = g.standard_normal((L, 2 * d)) * 0.1
+        b1 = g.standard_normal(L) * 0.1
+        W2 = (0 if zero else 1) * g.standard_normal((d, L)) * 0.1
+        b2 = (0 if zero else 1) * g.standard_normal(d) * 0.1
+        return W1, b1, W2, b2
+    return mlp(), mlp(delta_zero)
+
+
+def test_surrogate_mean_context_equals_uniform_routing_vector():
+    """Context replaced by the mean-pooled value vector = the surrogate with r_h = 1/N."""
+    g = np.random.default_rng(31)
+    N, d = 40, 64
+    V = g.standard_normal((N, d))
+    mg, md = _mlps(g)
+    r = g.dirichlet(np.ones(N))
+    got, C = oracle.surrogate_attention(V, r, mg, md, mean_context=True)
+    want, Cw = oracle.surrogate_attention(V, np.full(N, 1.0 / N), mg, md)
+    np.testing.assert_allclose(C, V.mean(0), rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-14)
+
+
+def test_surrogate_without_residual_equals_zero_delta_mlp():
+    """No token-wise residual correction: y_i = C_h, the same as a zero MLP_delta."""
+    g = np.random.default_rng(32)
+    N, d = 33, 64
+    V = g.standard_normal((N, d))
+    r = g.dirichlet(np.ones(N))
+    mg, md = _mlps(g, delta_zero=True)
+    got, C = oracle.surrogate_attention(V, r, mg, md, residual=False, rows=np.arange(5, 20))
+    want, _ = oracle.surrogate_attention(V, r, mg, md, rows=np.arange(5, 20))
+    np.testing.assert_allclose(got, np.tile(r @ V, (15, 1)), rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-14)
+
+
+def test_elu_feature_map():
+    x = np.array([-30.0, -2.0, -1e-9, 0.0, 1e-9, 0.5, 3.0])
+    want = np.array([np.exp(-30.0), np.exp(-2.0), np.exp(-1e-9), 1.0, 1.0 + 1e-9, 1.5, 4.0])
+    np.testing.assert_allclose(oracle.elu_feature_map(x), want, rtol=1e-15)
+    assert np.all(oracle.elu_feature_map(x) > 0)
+
+
+def test_linear_attention_closed_forms_and_brute_force():
+    g = np.random.default_rng(33)
+    N, d = 23, 64
+    Q, K, V = g.standard_normal((N, d)), g.standard_normal((N, d)), g.standard_normal((N, d))
+    # constant V rows give V back; identical keys give the mean of V for every query
+    c = g.standard_normal(d)
+    np.testing.assert_allclose(oracle.linear_attention(Q, K, np.tile(c, (N, 1))), np.tile(c, (N, 1)), rtol=1e-12)
+    np.testing.assert_allclose(oracle.linear_attention(Q, np.tile(K[0], (N, 1)), V), np.tile(V.mean(0), (N, 1)),
+                               rtol=1e-11, atol=1e-13)
+    # brute force, one pair at a time, from the elementwise feature map
+    phi = lambda x: x + 1.0 if x > 0 else np.exp(x)
+    out = oracle.linear_attention(Q, K, V, chunk=5)
+    for i in (0, 7, N - 1):
+        w = np.array([sum(phi(Q[i, t]) * phi(K[j, t]) for t in range(d)) for j in range(N)])
+        np.testing.assert_allclose(out[i], (w @ V) / w.sum(), rtol=1e-11)
+    # the factored order the kernels use, phi(Q) (phi(K)^T V) / (phi(Q) phi(K)^T 1), is the same map
+    fQ, fK = oracle.elu_feature_map(Q), oracle.elu_feature_map(K)
+    np.testing.assert_allclose(out, (fQ @ (fK.T @ V)) / (fQ @ fK.sum(0))[:, None], rtol=1e-11)
+    # positive weights: every output lies within the range of V's column
+    assert np.all(out <= V.max(0) + 1e-12) and np.all(out >= V.min(0) - 1e-12)
+    # rows subset
+    np.testing.assert_allclose(oracle.linear_attention(Q, K, V, rows=[3, 9]), out[[3, 9]], rtol=1e-13)

@@ -143,3 +143,23 @@ def test_bin_heads_is_a_stable_partition():
         # Brute force: every (full head, tile) pair exactly once, head-major.
         expect = [(h, t) for h in range(H) if modes[h] == MODE_FULL for t in range(n_tiles)]
         assert [tuple(x) for x in work.tolist()] == expect
+
+
+def test_mean_query_pooling_ablation():
+    """§5 component ablation: Q-Pooling replaced by mean pooling, independent of the weights."""
+    g = np.random.default_rng(41)
+    N, d = 37, 64
+    Q = g.standard_normal((N, d))
+    for _ in range(2):
+        W, U, w = g.standard_normal((64, d)), g.standard_normal((64, d)), g.standard_normal(64)
+        alpha, qp = oracle.attention_pool(Q, W, U, w, mean_pool=True)
+        np.testing.assert_allclose(alpha, np.full(N, 1.0 / N), rtol=1e-15)
+        np.testing.assert_allclose(qp, Q.mean(0), rtol=1e-12, atol=1e-15)
+
+
+def test_two_branch_routing_has_no_surrogate_band():
+    """§5 compute-mode ablation "mean + full only": tau_low == tau_high leaves no band."""
+    t = np.float32(0.05)
+    for s in np.float32([0.0, 0.01, 0.049, 0.05, 0.0500001, 0.3, 1.0]):
+        m = oracle.select_mode(s, t, t)
+        assert m == (oracle.MODE_FULL if s >= t else oracle.MODE_MEAN)
