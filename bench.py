@@ -378,6 +378,8 @@ def run_ours(args):
         line["full_attention_s100"] = full_attention_probe(vpb, dev, N, dws[0], pk)
     if args.s32:
         line["stack_s32"] = s32_probe(vpb, dev)
+    if args.variants:
+        line["cheap_mode_variants"] = variant_probe(vpb, dev, N, dws[0], pk)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
@@ -416,6 +418,45 @@ def s32_probe(vpb, dev, steps=3, warmup=2):
             "routing": "natural (untrained routers)", "ms_per_forward": ms,
             "views_per_s": wl.views / (ms / 1e3),
             "routes": {"mean": int((m == 0).sum()), "surrogate": int((m == 1).sum()), "full": int((m == 2).sum())}}
+
+
+def variant_probe(vpb, dev, N, dw, pk):
+    """The cheap head modes over N tokens with all 16 heads in one mode: the §4.3 surrogate,
+    its §5 ablations (no residual correction; linear attention, state pass included) and mean
+    pooling.  Rates are algorithmic bytes (a surrogate head reads V and writes Y: 256 B per
+    token; linear attention reads Q, K, V and writes Y: 512 B; mean writes Y: 128 B) over time,
+    against the measured copy bandwidth."""
+    import torch
+    qkv = torch.randn(N, 3 * D, device=dev).to(torch.bfloat16)
+    y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+    ids = torch.arange(H, dtype=torch.int32, device=dev)
+    ctx = torch.randn(H, d, device=dev) * 0.1
+    mv = torch.randn(H, d, device=dev) * 0.1
+    sw = vpb.surrogate_weights(dw)
+    hbm = pk.get("hbm_gbs") or 6784.8
+    out = {}
+    cases = [("surrogate", 0, [0, 0, H, H], 256), ("surrogate_no_residual", 4, [0, 0, H, H], 128),
+             ("linear_attention", 8, [0, 0, H, H], 512), ("mean", 0, [0, H, H, H], 128)]
+    for name, variant, offs, bytes_per_token in cases:
+        dm = vpb.dims(N, H, variant=variant)
+        ws = vpb.workspace(dm, vpb.VP_WS_ROUTER, dev)
+        off = torch.tensor(offs, dtype=torch.int32, device=dev)
+        for _ in range(2):
+            vpb.vp_head_attention(dm, qkv, ids, off, ctx, mv, sw, y, ws)
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(5):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            vpb.vp_head_attention(dm, qkv, ids, off, ctx, mv, sw, y, ws)
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        ms = float(np.median(ts))
+        gbs = bytes_per_token * N * H / (ms * 1e-3) / 1e9
+        out[name] = {"ms_16_heads": ms, "gb_s": gbs, "hbm_frac": gbs / hbm}
+    out["tokens"] = N
+    return out
 
 
 def full_attention_probe(vpb, dev, N, dw, pk):
@@ -531,6 +572,8 @@ def main():
     ap.add_argument("--no-full-layer", dest="full_layer", action="store_false")
     ap.add_argument("--s32", action="store_true", default=True)
     ap.add_argument("--no-s32", dest="s32", action="store_false")
+    ap.add_argument("--variants", action="store_true", default=True)
+    ap.add_argument("--no-variants", dest="variants", action="store_false")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "layer_norm", "router", "surrogate"],
                     default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")

@@ -69,8 +69,20 @@ typedef struct vp_dims {
   int32_t d;        /* head dim, must be 64 */
   int32_t L;        /* router and surrogate hidden width, must be 64 (App. B) */
   float tau_low;    /* 0.01 in the paper (§4.2) */
-  float tau_high;   /* 0.20 in the paper (§4.2) */
+  float tau_high;   /* 0.20 in the paper (§4.2); tau_low == tau_high gives the two-branch
+                       router of §5's compute-mode ablation (mean and full only) */
+  uint32_t variant; /* 0 = the method; else an OR of VP_VARIANT_* (§5 ablations) */
 } vp_dims;
+
+/* Ablation variants of §5 (vp_dims.variant).  Component ablation: */
+#define VP_VARIANT_MEAN_QPOOL 1u        /* router: mean of the queries instead of the gated
+                                           attention pooling (alpha = 1/N) */
+#define VP_VARIANT_MEAN_CONTEXT 2u      /* surrogate: C_h = mean of V_h instead of r_h V_h */
+#define VP_VARIANT_NO_RESIDUAL 4u       /* surrogate: y_i = C_h, no token-wise correction */
+/* Compute-mode ablation: surrogate heads run linear attention (Katharopoulos et al. 2020,
+   phi(x) = elu(x) + 1): y_i = phi(q_i)^T S_h / phi(q_i)^T z_h with S_h = sum_j phi(k_j) v_j^T,
+   z_h = sum_j phi(k_j).  Not combinable with MEAN_CONTEXT or NO_RESIDUAL. */
+#define VP_VARIANT_LINEAR_ATTENTION 8u
 
 /* Router parameters (§4.1), per head; all device pointers. */
 typedef struct vp_router_weights {
@@ -112,7 +124,7 @@ typedef struct vp_layer_weights {
 } vp_layer_weights;
 
 /* Workspace kinds for vp_workspace_size. */
-#define VP_WS_ROUTER 0   /* vp_router, vp_head_attention */
+#define VP_WS_ROUTER 0   /* vp_router, vp_head_attention (router scratch + linear-attention state) */
 #define VP_WS_LAYER 1    /* vp_moh_global_attention */
 #define VP_WS_STACK 2    /* vp_global_stack */
 

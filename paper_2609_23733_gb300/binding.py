@@ -20,6 +20,7 @@ VP_MODE_MEAN, VP_MODE_SURROGATE, VP_MODE_FULL = 0, 1, 2
 VP_WS_ROUTER, VP_WS_LAYER, VP_WS_STACK = 0, 1, 2
 VP_ACT_NONE, VP_ACT_GELU = 0, 1
 VP_DEVERR_WAIT_TIMEOUT, VP_DEVERR_NAN_SALIENCY = 1, 2
+VP_VARIANT_MEAN_QPOOL, VP_VARIANT_MEAN_CONTEXT, VP_VARIANT_NO_RESIDUAL, VP_VARIANT_LINEAR_ATTENTION = 1, 2, 4, 8
 KERNEL_CLASSES = ["gemm", "router_pool", "router_keys", "router_r", "bin_heads", "attn_full",
                   "surrogate", "mean", "layer_norm"]
 
@@ -36,7 +37,7 @@ class VPError(RuntimeError):
 
 class VpDims(Structure):
     _fields_ = [("N", c_int32), ("H", c_int32), ("d", c_int32), ("L", c_int32),
-                ("tau_low", c_float), ("tau_high", c_float)]
+                ("tau_low", c_float), ("tau_high", c_float), ("variant", c_uint32)]
 
 
 class VpRouterWeights(Structure):
@@ -126,8 +127,8 @@ def _stream(stream=None):
     return s.cuda_stream
 
 
-def dims(N, H=16, d=64, L=64, tau_low=0.01, tau_high=0.20) -> VpDims:
-    return VpDims(int(N), int(H), int(d), int(L), float(tau_low), float(tau_high))
+def dims(N, H=16, d=64, L=64, tau_low=0.01, tau_high=0.20, variant=0) -> VpDims:
+    return VpDims(int(N), int(H), int(d), int(L), float(tau_low), float(tau_high), int(variant))
 
 
 def router_weights(w: dict) -> VpRouterWeights:

@@ -135,6 +135,12 @@ vp_status check_dims(const vp_dims* dm) {
   if (dm->d != kHeadDim || dm->L != kHidden || dm->H < 1 || dm->H > kMaxHeads || dm->N < 1)
     return VP_ERR_UNSUPPORTED_SHAPE;
   if (!(dm->tau_low == dm->tau_low) || !(dm->tau_high == dm->tau_high)) return VP_ERR_INVALID_ARG;
+  const uint32_t known = VP_VARIANT_MEAN_QPOOL | VP_VARIANT_MEAN_CONTEXT | VP_VARIANT_NO_RESIDUAL |
+                         VP_VARIANT_LINEAR_ATTENTION;
+  if (dm->variant & ~known) return VP_ERR_INVALID_ARG;
+  if ((dm->variant & VP_VARIANT_LINEAR_ATTENTION) &&
+      (dm->variant & (VP_VARIANT_MEAN_CONTEXT | VP_VARIANT_NO_RESIDUAL)))
+    return VP_ERR_INVALID_ARG;  // those two modify the §4.3 surrogate, which linear attention replaces
   return VP_OK;
 }
 
@@ -145,13 +151,13 @@ vp_status check_device() {
 
 size_t layer_ws_bytes(const vp_dims* dm) {
   const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
-  return router_scratch_bytes(dm->H) + align_up(N * 3 * D * 2) + align_up(N * D * 2);
+  return heads_scratch_bytes(dm->H) + align_up(N * 3 * D * 2) + align_up(N * D * 2);
 }
 
 size_t stack_ws_bytes(const vp_dims* dm) {
   const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
   // x~ (LN output) + one region shared by {QKV, Y} and the FFN hidden layer.
-  return router_scratch_bytes(dm->H) + align_up(N * D * 2) + align_up(N * 4 * D * 2);
+  return heads_scratch_bytes(dm->H) + align_up(N * D * 2) + align_up(N * 4 * D * 2);
 }
 
 // Row widths the LayerNorm kernel is instantiated for.
@@ -189,6 +195,7 @@ RouterArgs make_router_args(const vp_dims* dm, const vp_bf16* qkv, const vp_rout
   a.H = dm->H;
   a.tau_low = dm->tau_low;
   a.tau_high = dm->tau_high;
+  a.variant = dm->variant;
   a.qkv = reinterpret_cast<const __nv_bfloat16*>(qkv);
   a.W = reinterpret_cast<const __nv_bfloat16*>(rw->W);
   a.U = reinterpret_cast<const __nv_bfloat16*>(rw->U);
@@ -224,8 +231,11 @@ vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* 
   ha.qkv = qkv;
   ha.head_ids = head_ids;
   ha.offsets = offsets;
-  ha.ctx = ctx;
+  // §5 component ablation "Context": the surrogate's context is the mean-pooled value vector.
+  ha.ctx = (dm->variant & VP_VARIANT_MEAN_CONTEXT) ? mean_v : ctx;
   ha.mean_v = mean_v;
+  ha.variant = dm->variant;
+  ha.lin_state = sc.lin_state;
   ha.sw = make_surrogate_args(sw);
   ha.y = y;
   ha.s_attn = s_attn;
@@ -302,7 +312,7 @@ vp_status vp_workspace_size(const vp_dims* dims, int32_t what, size_t* bytes) {
   VP_TRY(check_dims(dims));
   if (!bytes) return VP_ERR_INVALID_ARG;
   switch (what) {
-    case VP_WS_ROUTER: *bytes = router_scratch_bytes(dims->H); break;
+    case VP_WS_ROUTER: *bytes = heads_scratch_bytes(dims->H); break;
     case VP_WS_LAYER: *bytes = layer_ws_bytes(dims); break;
     case VP_WS_STACK: *bytes = stack_ws_bytes(dims); break;
     default: return VP_ERR_INVALID_ARG;
@@ -407,7 +417,7 @@ vp_status vp_head_attention(const vp_dims* dims, const vp_bf16* qkv, const int32
   if (!qkv || !head_ids || !offsets || !ctx || !mean_v || !y) return VP_ERR_INVALID_ARG;
   if (!aligned16(qkv) || !aligned16(y)) return VP_ERR_ALIGNMENT;
   VP_TRY(check_surrogate_weights(sw));
-  if (!ws || ws_bytes < router_scratch_bytes(dims->H)) return VP_ERR_WORKSPACE;
+  if (!ws || ws_bytes < heads_scratch_bytes(dims->H)) return VP_ERR_WORKSPACE;
   VP_TRY(check_device());
   RouterScratch sc = carve_router_scratch(ws, dims->H);
   return run_heads(dims, reinterpret_cast<const __nv_bfloat16*>(qkv), head_ids, offsets, ctx,
@@ -474,7 +484,7 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t N = dims->N, D = (size_t)dims->H * kHeadDim;
   RouterScratch sc = carve_router_scratch(ws, dims->H);
-  char* p = static_cast<char*>(ws) + router_scratch_bytes(dims->H);
+  char* p = static_cast<char*>(ws) + heads_scratch_bytes(dims->H);
   __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
   p += align_up(N * 3 * D * 2);
   __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p);
@@ -513,7 +523,7 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t N = dims->N;
   RouterScratch sc = carve_router_scratch(ws, dims->H);
-  char* p = static_cast<char*>(ws) + router_scratch_bytes(dims->H);
+  char* p = static_cast<char*>(ws) + heads_scratch_bytes(dims->H);
   __nv_bfloat16* xt = reinterpret_cast<__nv_bfloat16*>(p);
   p += align_up(N * D * 2);
   __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);

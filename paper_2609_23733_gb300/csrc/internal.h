@@ -35,14 +35,23 @@ struct RouterScratch {
   int32_t* head_ids;            // [H]
   int32_t* offsets;             // [4]
   unsigned int* cheap_counter;  // work counter of the cheap head modes
+  float* lin_state;             // [H][kLinState] linear-attention state (after the router part)
 };
 
+// Linear-attention state of one head (the §5 compute-mode ablation): S_h [64 c][64 e] =
+// sum_j phi(k_j)[c] v_j[e], then z_h [64] = sum_j phi(k_j), fp32.
+constexpr int kLinState = 64 * 64 + 64;
+
+// Bytes of the router's scratch (what vp_router touches).
 size_t router_scratch_bytes(int H);
+// Router scratch + linear-attention state: the workspace of the head modes.
+size_t heads_scratch_bytes(int H);
 RouterScratch carve_router_scratch(void* ws, int H);
 
 struct RouterArgs {
   int N, H;
   float tau_low, tau_high;
+  uint32_t variant;  // VP_VARIANT_* bits
   const __nv_bfloat16* qkv;
   const __nv_bfloat16* W;
   const __nv_bfloat16* U;
@@ -82,6 +91,8 @@ struct HeadAttnArgs {
   SurrogateArgs sw;
   __nv_bfloat16* y;
   float* s_attn;                // [H] MaxAttn saliency of the full heads, or NULL
+  uint32_t variant;             // VP_VARIANT_* bits
+  float* lin_state;             // [H][kLinState] (VP_VARIANT_LINEAR_ATTENTION only)
   unsigned int* err;
   unsigned int* cheap_counter;  // one word of scratch, zeroed by the launcher
 };

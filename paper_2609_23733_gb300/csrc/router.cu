@@ -60,6 +60,7 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
   const int h = blockIdx.y, split = blockIdx.x;
   const int N = a.N, H = a.H;
   const size_t row_pitch = (size_t)3 * H * kHeadDim;  // elements between consecutive tokens
+  const bool mean_pool = (a.variant & VP_VARIANT_MEAN_QPOOL) != 0;  // §5 component ablation
 
   __shared__ __align__(16) __nv_bfloat16 sB[128 * kBStride];  // rows 0..63 W_h, 64..127 U_h
   __shared__ float s_bias[128];                              // bW | bU
@@ -108,6 +109,9 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
       qb[0] = y0.x; qb[1] = y0.y; qb[2] = y0.z; qb[3] = y0.w;
       qb[4] = y1.x; qb[5] = y1.y; qb[6] = y1.z; qb[7] = y1.w;
     }
+    // Pooling logits (both 0 under the mean-pooling ablation: alpha = 1/N exactly).
+    float ea = 0.f, eb = 0.f;
+    if (!mean_pool) {
     float acc[16][4];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
@@ -123,7 +127,6 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
     }
     // Pooling logits: columns 8j + 2c + e of the W half (j < 8) pair with the same
     // columns of the U half (j + 8) in the same thread.
-    float ea = 0.f, eb = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
 #pragma unroll
@@ -137,6 +140,7 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
     ea += __shfl_xor_sync(0xffffffffu, ea, 2);
     eb += __shfl_xor_sync(0xffffffffu, eb, 1);
     eb += __shfl_xor_sync(0xffffffffu, eb, 2);
+    }
     if (!va) ea = -INFINITY;
     if (!vb) eb = -INFINITY;
     float mc = fmaxf(ea, eb);
@@ -453,6 +457,10 @@ size_t router_scratch_bytes(int H) {
   return (b + 4095) & ~(size_t)4095;
 }
 
+size_t heads_scratch_bytes(int H) {
+  return router_scratch_bytes(H) + (size_t)kMaxHeads * kLinState * 4;
+}
+
 RouterScratch carve_router_scratch(void* ws, int H) {
   (void)H;
   char* p = static_cast<char*>(ws);
@@ -480,6 +488,7 @@ RouterScratch carve_router_scratch(void* ws, int H) {
   sc.head_ids = reinterpret_cast<int32_t*>(p);
   sc.offsets = sc.head_ids + kMaxHeads;
   sc.cheap_counter = sc.counters + 96;  // counters[0 .. 2 * kMaxHeads] serve the router
+  sc.lin_state = reinterpret_cast<float*>(static_cast<char*>(ws) + router_scratch_bytes(H));
   return sc;
 }
 
