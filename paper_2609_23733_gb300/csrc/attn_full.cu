@@ -15,7 +15,10 @@
 //                 rescaled lazily: O and the sum are rescaled only when the max grows by
 //                 more than 2^8; otherwise the stale max is kept (exact either way).
 // While one chain's softmax runs, the tensor core works on the other chain's S and P V
-// products, and S_c(j+1) is issued as soon as chain c has read S_c(j).
+// products, and S_c(j+1) is issued as soon as chain c has read S_c(j).  The two chains' warps
+// on one SM sub-partition take turns at the exponentials (an mbarrier token per
+// sub-partition and chain): left alone they fall into step and share the MUFU for the whole
+// exponential phase, leaving it idle during the rest of the tile.
 // TMEM: S_0 [0,128) S_1 [128,256) O_0 [256,320) O_1 [320,384) P_0 [384,448) P_1 [448,512).
 // Keys past N are zero-filled by TMA and masked to -inf; query rows past N are not stored.
 // Optionally the epilogue also yields the head's MaxAttn saliency max_ij A_ij (§3).
@@ -49,6 +52,7 @@ struct FullSmem {
   uint64_t q_full, q_empty;
   uint64_t k_full[kStages], v_full[kStages], kv_empty[kStages];
   uint64_t s_full[2], s_empty[2], p_full[2], o_bar[2], o_empty[2], drain[2];
+  uint64_t mufu[2][4];  // [chain][SM sub-partition]: chain c's warp there finished its exponentials
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -95,6 +99,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sm.o_bar[c], 1);
       mbar_init(&sm.o_empty[c], 128);
       mbar_init(&sm.drain[c], 1);
+      for (int q = 0; q < 4; ++q) mbar_init(&sm.mufu[c][q], 1);
     }
     sm.abort_flag = 0;
     fence_mbarrier_init();
@@ -291,6 +296,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           alpha = fast_exp2(m - mx2);
           m = mx2;
         }
+        // The two chains' warps on this SM sub-partition take turns at the exponentials (MUFU):
+        // chain 1 waits for chain 0's tile g, chain 0 for chain 1's tile g - 1.
+        if (c == 1 || g > 0) {
+          ok = mbar_wait_warp(&sm.mufu[c ^ 1][quarter], c == 1 ? (g & 1) : ((g - 1) & 1), prm.err,
+                              abort_flag);
+          if (!ok) break;
+        }
         // p = 2^(s cs - m), summed in packed pairs and packed to bf16 pairs for P (before the
         // wait for P_c(g-1) V below, so that only the TMEM stores follow it).
         const float2 c2 = make_float2(cs, cs), nm = make_float2(-m, -m);
@@ -307,6 +319,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           else
             acc0 = fadd2(acc0, x);
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.mufu[c][quarter]);
         const float2 at = fadd2(acc0, acc1);
         lsum = lsum * alpha + (at.x + at.y);
         // P_c and O_c are free once P_c(g-1) V has completed.
