@@ -1,25 +1,28 @@
 // Full-mode heads (Algorithm 1, step 2, s_h >= tau_high): Y_h = softmax(Q_h K_h^T / sqrt d) V_h
 // as a flash-attention kernel on the sm_103a tensor cores.
 //
-// Persistent CTAs (one per SM) walk the work items (full head, pair of 128-query tiles)
-// read from the device bins.  The two query tiles of an item run as two independent
-// chains, c = 0 and c = 1, that share the K/V pipeline:
-//   warp 0        TMA producer: both Q tiles once per item, K/V tiles through a 4-stage ring.
-//   warp 1        TMEM owner.  Warps 1 and 2: one elected lane each issues chain c's tcgen05.mma:
-//                 S_c = Q_c K^T (SS form, 128 x 128 fp32 in TMEM) and O_c += P_c V
-//                 (TS form: P_c read from TMEM as bf16, V from shared memory, MN-major).
-//   warps 4-7     softmax of chain 0, warps 8-11 softmax of chain 1: one query row per
-//                 thread (its TMEM lane).  The thread loads its S row, takes the max (3-input
-//                 max), computes 2^(s c - m) (packed f32x2 FMA + MUFU ex2), sums with packed
-//                 adds, and writes P as bf16 pairs back to TMEM.  The running max is
-//                 rescaled lazily: O and the sum are rescaled only when the max grows by
-//                 more than 2^8; otherwise the stale max is kept (exact either way).
-// While one chain's softmax runs, the tensor core works on the other chain's S and P V
-// products, and S_c(j+1) is issued as soon as chain c has read S_c(j).  The two chains' warps
-// on one SM sub-partition take turns at the exponentials (an mbarrier token per
-// sub-partition and chain): left alone they fall into step and share the MUFU for the whole
-// exponential phase, leaving it idle during the rest of the tile.
-// TMEM: S_0 [0,128) S_1 [128,256) O_0 [256,320) O_1 [320,384) P_0 [384,448) P_1 [448,512).
+// Persistent CTAs (one per SM) walk the work items (full head, group of kChains 128-query
+// tiles) read from the device bins.  The query tiles of an item run as independent chains
+// c = 0 .. kChains-1 that share the K/V pipeline (kBN keys per tile):
+//   warp 0        TMA producer: the item's Q tiles once, K/V tiles through a kStages ring.
+//   warp 1        TMEM owner.  Warps 1 .. kChains: one elected lane each issues chain c's
+//                 tcgen05.mma: S_c = Q_c K^T (SS form, 128 x kBN fp32 in TMEM) and
+//                 O_c += P_c V (TS form: P_c read from TMEM as bf16, V from shared memory,
+//                 MN-major).
+//   warps 4 ..    four softmax warps per chain: one query row per thread (its TMEM lane).
+//                 The thread loads its S row, takes the max (3-input max), computes
+//                 2^(s c - m) (packed f32x2 FMA + MUFU ex2), sums with packed adds, and
+//                 writes P as bf16 pairs back to TMEM.  The running max is rescaled lazily:
+//                 O and the sum are rescaled only when the max grows by more than 2^8;
+//                 otherwise the stale max is kept (exact either way).
+// S_c(j+1) is issued as soon as chain c has read S_c(j), so the tensor core works on the
+// other chains while one chain's softmax runs.  The configuration (VP_ATTN_CHAINS,
+// VP_ATTN_BN) is 3 chains of 64-key tiles: every SM sub-partition then holds three softmax
+// warps, whose exponentials, maxima and TMEM traffic overlap (measured on GB300: 3 % faster
+// than 2 chains of 128-key tiles with 16 heads, 9 % with 2 heads).  Optionally
+// (VP_ATTN_MUFU_TURNS) the chains' warps on one sub-partition take turns at the exponentials
+// through an mbarrier token; that helps 2 chains, which otherwise fall into step, and hurts 3.
+// TMEM: S_c at [c kBN, +kBN), O_c at [kChains kBN + 64 c, +64), P_c after the O columns.
 // Keys past N are zero-filled by TMA and masked to -inf; query rows past N are not stored.
 // Optionally the epilogue also yields the head's MaxAttn saliency max_ij A_ij (§3).
 // Every CTA signals its dependents at once (griddepcontrol.launch_dependents), so the
@@ -36,23 +39,43 @@ namespace vp {
 
 namespace {
 
-constexpr int kBM = 128;       // query rows per tile (two tiles per item)
-constexpr int kBN = 128;       // keys per tile
-constexpr int kStages = 4;     // K/V ring depth
-constexpr int kTileBytes = 128 * 64 * 2;  // one 128 x 64 bf16 tile (16 KB)
+#ifndef VP_ATTN_CHAINS
+#define VP_ATTN_CHAINS 3
+#endif
+#ifndef VP_ATTN_BN
+#define VP_ATTN_BN 64
+#endif
+constexpr int kChains = VP_ATTN_CHAINS;  // query tiles (chains) per work item
+constexpr int kBM = 128;                 // query rows per tile
+constexpr int kBN = VP_ATTN_BN;          // keys per tile
+constexpr int kStages = 512 / kBN;       // K/V ring depth: 64 KB of K and 64 KB of V
+constexpr int kQTileBytes = kBM * 64 * 2;
+constexpr int kKVTileBytes = kBN * 64 * 2;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
+// TMEM: S_c (fp32, kBN columns), O_c (fp32, 64), P_c (bf16 pairs, kBN / 2) for every chain.
+constexpr uint32_t kColS = 0, kColO = kChains * kBN, kColP = kColO + kChains * 64;
+static_assert(kColP + kChains * kBN / 2 <= kTmemCols, "TMEM columns");
 constexpr float kRescaleThreshold = 8.f;  // log2 units
-constexpr int kThreads = 384;
+#ifndef VP_ATTN_MUFU_TURNS
+#define VP_ATTN_MUFU_TURNS 0
+#endif
+constexpr bool kMufuTurns = VP_ATTN_MUFU_TURNS != 0;
+constexpr int kThreads = 128 + 128 * kChains;
+// Register split (setmaxnreg): control warps drop, softmax warps rise, within the launch's
+// 65,536 registers: 128 x kCtrlRegs + 128 kChains x kSoftRegs <= 65,536.
+constexpr int kCtrlRegs = kChains == 3 ? 56 : 80;
+constexpr int kSoftRegs = kChains == 3 ? 152 : 208;
+static_assert(128 * kCtrlRegs + 128 * kChains * kSoftRegs <= 65536, "register split");
 
 struct FullSmem {
-  __nv_bfloat16 q[2][128 * 64];
-  __nv_bfloat16 k[kStages][128 * 64];
-  __nv_bfloat16 v[kStages][128 * 64];
+  __nv_bfloat16 q[kChains][kBM * 64];
+  __nv_bfloat16 k[kStages][kBN * 64];
+  __nv_bfloat16 v[kStages][kBN * 64];
   uint64_t q_full, q_empty;
   uint64_t k_full[kStages], v_full[kStages], kv_empty[kStages];
-  uint64_t s_full[2], s_empty[2], p_full[2], o_bar[2], o_empty[2], drain[2];
-  uint64_t mufu[2][4];  // [chain][SM sub-partition]: chain c's warp there finished its exponentials
+  uint64_t s_full[kChains], s_empty[kChains], p_full[kChains], o_bar[kChains], o_empty[kChains];
+  uint64_t drain[kChains];
+  uint64_t mufu[kChains][4];  // [chain][SM sub-partition]: that warp finished its exponentials
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -67,7 +90,8 @@ struct FullParams {
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
-    attn_full_kernel(const __grid_constant__ CUtensorMap tmap_qkv, FullParams prm) {
+    attn_full_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                     const __grid_constant__ CUtensorMap tmap_kv, FullParams prm) {
   extern __shared__ unsigned char smem_raw[];
   FullSmem& sm = *reinterpret_cast<FullSmem*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -75,9 +99,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int first = __ldg(prm.offsets + 2);
   const int n_heads = __ldg(prm.offsets + 3) - first;
   const int N = prm.N, H = prm.H;
-  const int n_pairs = (N + 2 * kBM - 1) / (2 * kBM);
+  const int n_groups = (N + kChains * kBM - 1) / (kChains * kBM);  // query-tile groups per head
   const int n_kv = (N + kBN - 1) / kBN;
-  const int items = n_heads * n_pairs;
+  const int items = n_heads * n_groups;
   if ((int)blockIdx.x >= items) return;  // uniform across the CTA
 
   const int warp = warp_uniform_id(), lane = lane_id();
@@ -86,13 +110,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
-    mbar_init(&sm.q_empty, 2);
+    mbar_init(&sm.q_empty, kChains);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 2);
+      mbar_init(&sm.kv_empty[s], kChains);
     }
-    for (int c = 0; c < 2; ++c) {
+    for (int c = 0; c < kChains; ++c) {
       mbar_init(&sm.s_full[c], 1);
       mbar_init(&sm.s_empty[c], 128);
       mbar_init(&sm.p_full[c], 128);
@@ -104,7 +128,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm.abort_flag = 0;
     fence_mbarrier_init();
     fence_proxy_async_smem();
-    tma_prefetch_desc(&tmap_qkv);
+    tma_prefetch_desc(&tmap_q);
+    tma_prefetch_desc(&tmap_kv);
   }
   if (warp == 1) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
@@ -115,11 +140,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
 
-  // Register split (setmaxnreg, per warpgroup): the control warpgroup (warps 0-3) drops to
-  // 80 registers, the two softmax warpgroups rise to 208: 80 x 128 + 208 x 256 = 63,488 <=
-  // 168 x 384, the allocation the CTA is launched with.
   if (warp < 4) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 80;");
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kCtrlRegs));
   }
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -128,14 +150,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t lc = 0, ic = 0;
     bool ok = true;
     for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
-      const int h = __shfl_sync(0xffffffffu, __ldg(prm.head_ids + first + item / n_pairs), 0);
-      const int qp = item % n_pairs;
+      const int h = __shfl_sync(0xffffffffu, __ldg(prm.head_ids + first + item / n_groups), 0);
+      const int qg = item % n_groups;
       ok = mbar_wait_warp(&sm.q_empty, (ic & 1) ^ 1, prm.err, abort_flag);
       if (!ok) break;
       if (elect_one()) {
-        mbar_arrive_expect_tx(&sm.q_full, 2 * kTileBytes);
-        tma_load_2d(sm.q[0], &tmap_qkv, &sm.q_full, h * 64, qp * 2 * kBM);
-        tma_load_2d(sm.q[1], &tmap_qkv, &sm.q_full, h * 64, qp * 2 * kBM + kBM);
+        mbar_arrive_expect_tx(&sm.q_full, kChains * kQTileBytes);
+#pragma unroll
+        for (int c = 0; c < kChains; ++c)
+          tma_load_2d(sm.q[c], &tmap_q, &sm.q_full, h * 64, (qg * kChains + c) * kBM);
       }
       __syncwarp();
       for (int j = 0; j < n_kv; ++j, ++lc) {
@@ -143,10 +166,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = mbar_wait_warp(&sm.kv_empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
         if (!ok) break;
         if (elect_one()) {
-          mbar_arrive_expect_tx(&sm.k_full[st], kTileBytes);
-          tma_load_2d(sm.k[st], &tmap_qkv, &sm.k_full[st], (H + h) * 64, j * kBN);
-          mbar_arrive_expect_tx(&sm.v_full[st], kTileBytes);
-          tma_load_2d(sm.v[st], &tmap_qkv, &sm.v_full[st], (2 * H + h) * 64, j * kBN);
+          mbar_arrive_expect_tx(&sm.k_full[st], kKVTileBytes);
+          tma_load_2d(sm.k[st], &tmap_kv, &sm.k_full[st], (H + h) * 64, j * kBN);
+          mbar_arrive_expect_tx(&sm.v_full[st], kKVTileBytes);
+          tma_load_2d(sm.v[st], &tmap_kv, &sm.v_full[st], (2 * H + h) * 64, j * kBN);
         }
         __syncwarp();
       }
@@ -167,7 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 1 || warp == 2) {
+  } else if (warp <= kChains) {
     // ------------------------------------------------------------ MMA issuers (chain c)
     // Converged warp; the elected lane (the same lane every time: elect.sync picks the
     // lowest active lane) issues the MMAs and the commits that track them.
@@ -177,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t dq = sdesc_sw128(smem_u32(sm.q[c]));
     const uint32_t t_s = tmem + kColS + c * kBN;
     const uint32_t t_o = tmem + kColO + c * 64;
-    const uint32_t t_p = tmem + kColP + c * 64;
+    const uint32_t t_p = tmem + kColP + c * (kBN / 2);
     uint32_t lc = 0, ic = 0, g = 0;  // K/V tiles seen, items, S/P/O tiles of this chain
     bool ok = true;
     for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
@@ -218,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint64_t dv = sdesc_sw128(smem_u32(sm.v[st]));
         if (elect_one()) {
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk)  // 8 x K=16 covers 128 keys: 8 TMEM columns, 2 KB of V
+          for (int kk = 0; kk < kBN / 16; ++kk)  // K=16 keys per step: 8 TMEM columns, 2 KB of V
             tc_mma_ts(t_o, t_p + 8 * kk, dv + (uint64_t)(kk * 128), id_o,
                       (j > 0 || kk > 0) ? 1u : 0u);
           tc_commit(&sm.o_bar[c]);
@@ -238,21 +261,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax / epilogue
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 208;");
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kSoftRegs));
     const int c = (warp - 4) >> 2;  // chain
     const int quarter = warp & 3;   // TMEM lane quarter this warp may access
     const int row_in_tile = quarter * 32 + lane;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const uint32_t t_s = tmem + lane_off + kColS + c * kBN;
     const uint32_t t_o = tmem + lane_off + kColO + c * 64;
-    const uint32_t t_p = tmem + lane_off + kColP + c * 64;
+    const uint32_t t_p = tmem + lane_off + kColP + c * (kBN / 2);
     const float cs = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
     const int n_tail = N - (n_kv - 1) * kBN;        // valid keys in the last tile
     uint32_t g = 0;
     bool ok = true;
     for (int item = blockIdx.x; item < items && ok; item += gridDim.x) {
-      const int h = __ldg(prm.head_ids + first + item / n_pairs);
-      const int qp = item % n_pairs;
+      const int h = __ldg(prm.head_ids + first + item / n_groups);
+      const int qg = item % n_groups;
       // m: the (lazily updated) reference the exponentials are taken against; xmax: the
       // true running maximum of the row's scaled scores, for the MaxAttn saliency.
       float m = 0.f, lsum = 0.f, xmax = 0.f;
@@ -260,15 +283,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = mbar_wait_warp(&sm.s_full[c], g & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
-        float s[128];
+        float s[kBN];
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) tmem_ld32(t_s + 32 * cc, s + 32 * cc);
+        for (int cc = 0; cc < kBN / 32; ++cc) tmem_ld32(t_s + 32 * cc, s + 32 * cc);
         tmem_wait_ld();
         tc_fence_before();
         mbar_arrive(&sm.s_empty[c]);  // the MMA warp may overwrite S_c now
         if (j == n_kv - 1 && n_tail < kBN) {
 #pragma unroll
-          for (int i = 0; i < 128; ++i)
+          for (int i = 0; i < kBN; ++i)
             if (i >= n_tail) s[i] = -INFINITY;
         }
         // Row max: eight independent 3-input max chains, then a short tree.
@@ -279,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 8; ++k) t[k] = fmaxf(s[k], s[8 + k]);
 #pragma unroll
-          for (int i = 16; i < 128; i += 16) {
+          for (int i = 16; i < kBN; i += 16) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) t[k] = fmax3(t[k], s[i + k], s[i + 8 + k]);
           }
@@ -296,20 +319,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           alpha = fast_exp2(m - mx2);
           m = mx2;
         }
-        // The two chains' warps on this SM sub-partition take turns at the exponentials (MUFU):
-        // chain 1 waits for chain 0's tile g, chain 0 for chain 1's tile g - 1.
-        if (c == 1 || g > 0) {
-          ok = mbar_wait_warp(&sm.mufu[c ^ 1][quarter], c == 1 ? (g & 1) : ((g - 1) & 1), prm.err,
-                              abort_flag);
+        // Optional turns at the exponentials (MUFU) for the chains' warps on this SM
+        // sub-partition, in chain order: chain c > 0 waits for chain c - 1's tile g, chain 0
+        // for the last chain's tile g - 1.
+        if (kMufuTurns && (c > 0 || g > 0)) {
+          ok = mbar_wait_warp(&sm.mufu[c > 0 ? c - 1 : kChains - 1][quarter],
+                              c > 0 ? (g & 1) : ((g - 1) & 1), prm.err, abort_flag);
           if (!ok) break;
         }
         // p = 2^(s cs - m), summed in packed pairs and packed to bf16 pairs for P (before the
         // wait for P_c(g-1) V below, so that only the TMEM stores follow it).
         const float2 c2 = make_float2(cs, cs), nm = make_float2(-m, -m);
         float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
-        uint32_t pk[64];
+        uint32_t pk[kBN / 2];
 #pragma unroll
-        for (int i = 0; i < 64; ++i) {
+        for (int i = 0; i < kBN / 2; ++i) {
           float2 x = ffma2(make_float2(s[2 * i], s[2 * i + 1]), c2, nm);
           x.x = fast_exp2(x.x);
           x.y = fast_exp2(x.y);
@@ -319,8 +343,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           else
             acc0 = fadd2(acc0, x);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.mufu[c][quarter]);
+        if (kMufuTurns) {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.mufu[c][quarter]);
+        }
         const float2 at = fadd2(acc0, acc1);
         lsum = lsum * alpha + (at.x + at.y);
         // P_c and O_c are free once P_c(g-1) V has completed.
@@ -330,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
         }
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) tmem_st16(t_p + 16 * cc, pk + 16 * cc);
+        for (int cc = 0; cc < kBN / 32; ++cc) tmem_st16(t_p + 16 * cc, pk + 16 * cc);
         if (__any_sync(0xffffffffu, need)) {
           float o[64];
           tmem_ld32(t_o, o);
@@ -356,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(&sm.o_empty[c]);
-      const int row = qp * 2 * kBM + c * kBM + row_in_tile;
+      const int row = (qg * kChains + c) * kBM + row_in_tile;
       const float inv = 1.f / lsum;
       if (row < N) {
         uint4* dst = reinterpret_cast<uint4*>(prm.y + ((size_t)row * H + h) * 64);
@@ -394,15 +420,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
-  CUtensorMap tmap;
-  cudaError_t e = make_tmap_bf16_2d(&tmap, a.qkv, (uint64_t)3 * a.H * 64, (uint64_t)a.N,
-                                    (uint64_t)3 * a.H * 64, 64, 128);
+  CUtensorMap tmap_q, tmap_kv;  // boxes of 128 query rows / kBN key rows, 64 channels
+  cudaError_t e = make_tmap_bf16_2d(&tmap_q, a.qkv, (uint64_t)3 * a.H * 64, (uint64_t)a.N,
+                                    (uint64_t)3 * a.H * 64, 64, kBM);
+  if (e != cudaSuccess) return e;
+  e = make_tmap_bf16_2d(&tmap_kv, a.qkv, (uint64_t)3 * a.H * 64, (uint64_t)a.N,
+                        (uint64_t)3 * a.H * 64, 64, kBN);
   if (e != cudaSuccess) return e;
   const int smem = (int)sizeof(FullSmem) + 1024;
   e = cudaFuncSetAttribute(attn_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.s_attn, a.err};
-  attn_full_kernel<<<num_sms, kThreads, smem, st>>>(tmap, prm);
+  attn_full_kernel<<<num_sms, kThreads, smem, st>>>(tmap_q, tmap_kv, prm);
   return cudaGetLastError();
 }
 
