@@ -236,6 +236,9 @@ vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* 
   ha.mean_v = mean_v;
   ha.variant = dm->variant;
   ha.lin_state = sc.lin_state;
+  ha.fa_part = sc.fa_part;
+  ha.fa_stats = sc.fa_stats;
+  ha.fa_count = sc.fa_count;
   ha.sw = make_surrogate_args(sw);
   ha.y = y;
   ha.s_attn = s_attn;

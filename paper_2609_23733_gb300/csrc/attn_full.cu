@@ -86,9 +86,148 @@ struct FullParams {
   const int32_t* offsets;
   __nv_bfloat16* y;
   float* s_attn;  // [H] MaxAttn saliency (zeroed by the launcher), or NULL
+  float* part;    // split-tail partial O, (m, l, xmax) and arrival counters (zeroed)
+  float* stats;
+  unsigned int* count;
   unsigned int* err;
 };
 
+// The work of one launch: G groups (head, kChains query tiles) over P persistent CTAs.  The
+// first R = floor(G / P) rounds take whole groups; the T = G - R P groups of the last round
+// are split along the keys into S = floor(P / T) parts (at most the number of key tiles),
+// so that T S <= P CTAs share that round instead of T.  Unit u < R P is group u; unit
+// R P + S t + s is part s of group R P + t.
+struct Plan {
+  int R, T, S, units, whole;  // whole: units that are whole groups (they come first)
+};
+
+__device__ __forceinline__ Plan make_plan(int G, int P, int n_kv) {
+  Plan pl;
+  pl.R = G / P;
+  pl.T = G - pl.R * P;
+  pl.S = pl.T > 0 ? P / pl.T : 1;
+  if (pl.S > n_kv) pl.S = n_kv;
+  if (pl.S < 2 || pl.T * pl.S > kFaTailUnits) pl.S = 1;
+  pl.units = pl.S == 1 ? G : pl.R * P + pl.T * pl.S;
+  pl.whole = pl.S == 1 ? G : pl.R * P;
+  return pl;
+}
+
+struct Unit {
+  int group;       // head slot * n_groups + query-tile group
+  int j0, nk;      // key tiles [j0, j0 + nk)
+  int slot;        // split-tail slot (t S + s), -1 for a whole group
+  int tail;        // t
+};
+
+__device__ __forceinline__ Unit whole_unit(int u, int n_kv) {
+  Unit w;
+  w.group = u;
+  w.j0 = 0;
+  w.nk = n_kv;
+  w.slot = -1;
+  w.tail = -1;
+  return w;
+}
+
+__device__ __forceinline__ Unit unit_of(const Plan& pl, int u, int P, int n_kv) {
+  Unit w;
+  if (pl.S == 1 || u < pl.R * P) {
+    w.group = u;
+    w.j0 = 0;
+    w.nk = n_kv;
+    w.slot = -1;
+    w.tail = -1;
+  } else {
+    const int v = u - pl.R * P, t = v / pl.S, sp = v - t * pl.S;
+    w.group = pl.R * P + t;
+    w.j0 = sp * n_kv / pl.S;
+    w.nk = (sp + 1) * n_kv / pl.S - w.j0;
+    w.slot = v;
+    w.tail = t;
+  }
+  return w;
+}
+
+// Split-tail epilogue of one warp (32 rows of chain c, TMEM lanes at t_o): reads the part's
+// unnormalised O rows, releases O_c (o_empty), and publishes them with (m, l, xmax); the last
+// part of this (group, chain, lane quarter) to arrive combines all parts, M = max m_s,
+// O = sum 2^(m_s - M) O_s, l = sum 2^(m_s - M) l_s, and stores Y and the saliency.  Not
+// inlined, and given only values: the attention loop's code and registers stay as they are
+// without it.
+__device__ __noinline__ void split_part(FullParams prm, Plan plan, Unit w, int c, int quarter,
+                                        int lane, int row_in_tile, int row, int h, uint32_t t_o,
+                                        uint64_t* o_empty, float m, float lsum, float xmax) {
+  float o[64];
+  tmem_ld32(t_o, o);
+  tmem_ld32(t_o + 32, o + 32);
+  tmem_wait_ld();
+  tc_fence_before();
+  mbar_arrive(o_empty);
+  const size_t prow = (size_t)(w.slot * 4 + c) * kBM + row_in_tile;
+  float4* po = reinterpret_cast<float4*>(prm.part + prow * 64);
+#pragma unroll
+  for (int q = 0; q < 16; ++q) po[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+  reinterpret_cast<float4*>(prm.stats)[prow] = make_float4(m, lsum, xmax, 0.f);
+  __threadfence();
+  __syncwarp();
+  unsigned int last = 0;
+  if (lane == 0)
+    last = atomicAdd(prm.count + (w.tail * 4 + c) * 4 + quarter, 1u) == (unsigned)(plan.S - 1);
+  if (!__shfl_sync(0xffffffffu, last, 0)) return;
+  __threadfence();
+  const int slot0 = w.tail * plan.S;
+  float M = -INFINITY, X = -INFINITY;
+  for (int sp = 0; sp < plan.S; ++sp) {
+    const float4 st4 = __ldcg(reinterpret_cast<const float4*>(prm.stats) +
+                              (size_t)((slot0 + sp) * 4 + c) * kBM + row_in_tile);
+    M = fmaxf(M, st4.x);
+    X = fmaxf(X, st4.z);
+  }
+  float L = 0.f;
+#pragma unroll
+  for (int i = 0; i < 64; ++i) o[i] = 0.f;
+  for (int sp = 0; sp < plan.S; ++sp) {
+    const size_t qrow = (size_t)((slot0 + sp) * 4 + c) * kBM + row_in_tile;
+    const float4 st4 = __ldcg(reinterpret_cast<const float4*>(prm.stats) + qrow);
+    const float wgt = fast_exp2(st4.x - M);
+    L = fmaf(wgt, st4.y, L);
+    const float4* pq = reinterpret_cast<const float4*>(prm.part + qrow * 64);
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      const float4 f = __ldcg(pq + q);
+      o[4 * q] = fmaf(wgt, f.x, o[4 * q]);
+      o[4 * q + 1] = fmaf(wgt, f.y, o[4 * q + 1]);
+      o[4 * q + 2] = fmaf(wgt, f.z, o[4 * q + 2]);
+      o[4 * q + 3] = fmaf(wgt, f.w, o[4 * q + 3]);
+    }
+  }
+  const float inv = 1.f / L;
+  if (row < prm.N) {
+    uint4* dst = reinterpret_cast<uint4*>(prm.y + ((size_t)row * prm.H + h) * 64);
+#pragma unroll
+    for (int ch = 0; ch < 8; ++ch) {
+      uint4 v;
+      v.x = pack_bf16x2(o[8 * ch + 0] * inv, o[8 * ch + 1] * inv);
+      v.y = pack_bf16x2(o[8 * ch + 2] * inv, o[8 * ch + 3] * inv);
+      v.z = pack_bf16x2(o[8 * ch + 4] * inv, o[8 * ch + 5] * inv);
+      v.w = pack_bf16x2(o[8 * ch + 6] * inv, o[8 * ch + 7] * inv);
+      dst[ch] = v;
+    }
+  }
+  if (prm.s_attn) {
+    float a = row < prm.N ? fast_exp2(X - M) * inv : 0.f;
+#pragma unroll
+    for (int k = 16; k > 0; k >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, k));
+    if (lane == 0) atomicMax(reinterpret_cast<int*>(prm.s_attn + h), __float_as_int(a));
+  }
+}
+
+// kParts = false: the whole groups (all of them when nothing is split); kParts = true: the
+// split parts, one per CTA, launched right behind (programmatic dependent launch) so that
+// they take the SMs the whole groups leave.  Two instantiations keep runtime key ranges out
+// of the main one's attention loop, which they would slow down by about a tenth.
+template <bool kParts>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_full_kernel(const __grid_constant__ CUtensorMap tmap_q,
                      const __grid_constant__ CUtensorMap tmap_kv, FullParams prm) {
@@ -101,8 +240,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int N = prm.N, H = prm.H;
   const int n_groups = (N + kChains * kBM - 1) / (kChains * kBM);  // query-tile groups per head
   const int n_kv = (N + kBN - 1) / kBN;
-  const int items = n_heads * n_groups;
-  if ((int)blockIdx.x >= items) return;  // uniform across the CTA
+  const int P = gridDim.x;
+  const Plan plan = make_plan(n_heads * n_groups, P, n_kv);
+  // Units of this CTA: [u_begin, u_end) in steps of P.
+  const int u_begin = kParts ? plan.whole + (int)blockIdx.x : (int)blockIdx.x;
+  const int u_end = kParts ? (u_begin < plan.units ? u_begin + 1 : u_begin) : plan.whole;
+  if (u_begin >= u_end) {  // uniform across the CTA
+    // The parts grid completes only after the whole-group grid (its prerequisite): work
+    // queued behind it then sees every row of Y.
+    if (kParts && blockIdx.x == 0) {
+      asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+      asm volatile("griddepcontrol.wait;" ::: "memory");
+    }
+    return;
+  }
 
   const int warp = warp_uniform_id(), lane = lane_id();
   volatile int* abort_flag = &sm.abort_flag;
@@ -149,9 +300,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // one elected lane issues the copies.
     uint32_t lc = 0, ic = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
-      const int h = __shfl_sync(0xffffffffu, __ldg(prm.head_ids + first + item / n_groups), 0);
-      const int qg = item % n_groups;
+    for (int u = u_begin; u < u_end && ok; u += P, ++ic) {
+      const Unit w = kParts ? unit_of(plan, u, P, n_kv) : whole_unit(u, n_kv);
+      const int h = __shfl_sync(0xffffffffu, __ldg(prm.head_ids + first + w.group / n_groups), 0);
+      const int qg = w.group % n_groups;
       ok = mbar_wait_warp(&sm.q_empty, (ic & 1) ^ 1, prm.err, abort_flag);
       if (!ok) break;
       if (elect_one()) {
@@ -161,8 +313,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(sm.q[c], &tmap_q, &sm.q_full, h * 64, (qg * kChains + c) * kBM);
       }
       __syncwarp();
-      for (int j = 0; j < n_kv; ++j, ++lc) {
-        const int st = lc % kStages;
+      for (int jj = 0; jj < w.nk; ++jj, ++lc) {
+        const int j = w.j0 + jj, st = lc % kStages;
         ok = mbar_wait_warp(&sm.kv_empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
         if (!ok) break;
         if (elect_one()) {
@@ -201,9 +353,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_s = tmem + kColS + c * kBN;
     const uint32_t t_o = tmem + kColO + c * 64;
     const uint32_t t_p = tmem + kColP + c * (kBN / 2);
-    uint32_t lc = 0, ic = 0, g = 0;  // K/V tiles seen, items, S/P/O tiles of this chain
+    uint32_t lc = 0, ic = 0, g = 0;  // K/V tiles seen, units, S/P/O tiles of this chain
     bool ok = true;
-    for (int item = blockIdx.x; item < items && ok; item += gridDim.x, ++ic) {
+    const int n_kv_all = n_kv;
+    for (int u = u_begin; u < u_end && ok; u += P, ++ic) {
+      const int n_kv = kParts ? unit_of(plan, u, P, n_kv_all).nk : n_kv_all;  // tiles of this unit
       ok = mbar_wait_warp(&sm.q_full, ic & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
@@ -273,13 +427,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_tail = N - (n_kv - 1) * kBN;        // valid keys in the last tile
     uint32_t g = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < items && ok; item += gridDim.x) {
-      const int h = __ldg(prm.head_ids + first + item / n_groups);
-      const int qg = item % n_groups;
+    for (int u = u_begin; u < u_end && ok; u += P) {
+      const Unit w = kParts ? unit_of(plan, u, P, n_kv) : whole_unit(u, n_kv);
+      const int h = __ldg(prm.head_ids + first + w.group / n_groups);
+      const int qg = w.group % n_groups;
       // m: the (lazily updated) reference the exponentials are taken against; xmax: the
       // true running maximum of the row's scaled scores, for the MaxAttn saliency.
       float m = 0.f, lsum = 0.f, xmax = 0.f;
-      for (int j = 0; j < n_kv; ++j, ++g) {
+      for (int jj = 0; jj < w.nk; ++jj, ++g) {
+        const int j = w.j0 + jj;  // key tile
         ok = mbar_wait_warp(&sm.s_full[c], g & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
@@ -309,10 +465,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           mx = fmaxf(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], fmax3(t[5], t[6], t[7])));
         }
         const float mx2 = mx * cs;
-        xmax = j == 0 ? mx2 : fmaxf(xmax, mx2);
+        xmax = jj == 0 ? mx2 : fmaxf(xmax, mx2);
         float alpha = 1.f;
         bool need = false;
-        if (j == 0) {
+        if (jj == 0) {
           m = mx2;
         } else if (mx2 > m + kRescaleThreshold) {
           need = true;
@@ -376,13 +532,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = mbar_wait_warp(&sm.o_bar[c], (g - 1) & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
+      const int row = (qg * kChains + c) * kBM + row_in_tile;
+      if (kParts) {  // a part of a split group (the last round's groups)
+        split_part(prm, plan, w, c, quarter, lane, row_in_tile, row, h, t_o, &sm.o_empty[c], m,
+                   lsum, xmax);
+        __syncwarp();
+        continue;
+      }
       float o[64];
       tmem_ld32(t_o, o);
       tmem_ld32(t_o + 32, o + 32);
       tmem_wait_ld();
       tc_fence_before();
       mbar_arrive(&sm.o_empty[c]);
-      const int row = (qg * kChains + c) * kBM + row_in_tile;
       const float inv = 1.f / lsum;
       if (row < N) {
         uint4* dst = reinterpret_cast<uint4*>(prm.y + ((size_t)row * H + h) * 64);
@@ -415,6 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  if (kParts && blockIdx.x == 0 && threadIdx.x == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 }  // namespace
@@ -428,10 +591,29 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
                         (uint64_t)3 * a.H * 64, 64, kBN);
   if (e != cudaSuccess) return e;
   const int smem = (int)sizeof(FullSmem) + 1024;
-  e = cudaFuncSetAttribute(attn_full_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  e = cudaFuncSetAttribute(attn_full_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.s_attn, a.err};
-  attn_full_kernel<<<num_sms, kThreads, smem, st>>>(tmap_q, tmap_kv, prm);
+  e = cudaFuncSetAttribute(attn_full_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  FullParams prm{a.N, a.H, a.head_ids, a.offsets, a.y, a.s_attn, a.fa_part, a.fa_stats,
+                 a.fa_count, a.err};
+  attn_full_kernel<false><<<num_sms, kThreads, smem, st>>>(tmap_q, tmap_kv, prm);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  // The split parts of the last round (if the bins give one), on the SMs the whole groups free.
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(num_sms);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, attn_full_kernel<true>, tmap_q, tmap_kv, prm);
+  prof_extra_launch();
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -154,6 +154,8 @@ __global__ void __launch_bounds__(kThreads, 3) cheap_heads_kernel(HeadAttnArgs a
 cudaError_t launch_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(a.cheap_counter, 0, sizeof(unsigned int), st);
   if (e != cudaSuccess) return e;
+  e = cudaMemsetAsync(a.fa_count, 0, sizeof(unsigned int) * kFaCountWords, st);
+  if (e != cudaSuccess) return e;
   if (a.s_attn) {  // 0 for the heads that are not in full mode; full heads max into it
     e = cudaMemsetAsync(a.s_attn, 0, sizeof(float) * a.H, st);
     if (e != cudaSuccess) return e;

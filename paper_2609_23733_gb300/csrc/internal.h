@@ -36,7 +36,18 @@ struct RouterScratch {
   int32_t* offsets;             // [4]
   unsigned int* cheap_counter;  // work counter of the cheap head modes
   float* lin_state;             // [H][kLinState] linear-attention state (after the router part)
+  float* fa_part;               // [kFaTailUnits][4 chains][128 rows][64] split-tail partial O
+  float* fa_stats;              // [kFaTailUnits][4 chains][128 rows][4] (m, l, xmax, -)
+  unsigned int* fa_count;       // [kFaTailUnits][4 chains][4 quarters] split arrivals
 };
+
+// Full attention splits the work items of its last, partial round along the keys over the
+// CTAs that would otherwise idle; the partial results need this much scratch (units = groups
+// x splits of that round, at most one per CTA).
+constexpr int kFaTailUnits = 256;
+constexpr size_t kFaPartFloats = (size_t)kFaTailUnits * 4 * 128 * 64;
+constexpr size_t kFaStatsFloats = (size_t)kFaTailUnits * 4 * 128 * 4;
+constexpr size_t kFaCountWords = (size_t)kFaTailUnits * 4 * 4;
 
 // Linear-attention state of one head (the §5 compute-mode ablation): S_h [64 c][64 e] =
 // sum_j phi(k_j)[c] v_j[e], then z_h [64] = sum_j phi(k_j), fp32.
@@ -93,6 +104,9 @@ struct HeadAttnArgs {
   float* s_attn;                // [H] MaxAttn saliency of the full heads, or NULL
   uint32_t variant;             // VP_VARIANT_* bits
   float* lin_state;             // [H][kLinState] (VP_VARIANT_LINEAR_ATTENTION only)
+  float* fa_part;               // split-tail scratch of the full-attention kernel
+  float* fa_stats;
+  unsigned int* fa_count;       // zeroed by the launcher
   unsigned int* err;
   unsigned int* cheap_counter;  // one word of scratch, zeroed by the launcher
 };

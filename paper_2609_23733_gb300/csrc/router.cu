@@ -458,7 +458,8 @@ size_t router_scratch_bytes(int H) {
 }
 
 size_t heads_scratch_bytes(int H) {
-  return router_scratch_bytes(H) + (size_t)kMaxHeads * kLinState * 4;
+  return router_scratch_bytes(H) + (size_t)kMaxHeads * kLinState * 4 +
+         (kFaPartFloats + kFaStatsFloats + kFaCountWords) * 4;
 }
 
 RouterScratch carve_router_scratch(void* ws, int H) {
@@ -489,6 +490,9 @@ RouterScratch carve_router_scratch(void* ws, int H) {
   sc.offsets = sc.head_ids + kMaxHeads;
   sc.cheap_counter = sc.counters + 96;  // counters[0 .. 2 * kMaxHeads] serve the router
   sc.lin_state = reinterpret_cast<float*>(static_cast<char*>(ws) + router_scratch_bytes(H));
+  sc.fa_part = sc.lin_state + (size_t)kMaxHeads * kLinState;
+  sc.fa_stats = sc.fa_part + kFaPartFloats;
+  sc.fa_count = reinterpret_cast<unsigned int*>(sc.fa_stats + kFaStatsFloats);
   return sc;
 }
 
