@@ -380,3 +380,26 @@ def test_layer_s8_518_calibrated():
     np.testing.assert_array_equal(modes, want["modes"])
     np.testing.assert_allclose(s, want["s"], rtol=5e-3)
     compare(got[rows], want["out"], what="layer out (sampled rows)")
+
+
+def test_full_attention_split_tail_full_size():
+    """S = 100 views at 518 px (137,400 tokens), one full head among cheap ones, as in most
+    layers of the stack: on 152 SMs the last round's groups are split along the keys and
+    recombined.  Sampled rows from whole groups and from split groups against the oracle."""
+    N, H = 137400, 16
+    g = np.random.default_rng(137)
+    qkv = g.standard_normal((N, 3, H, 64)).astype(np.float32)
+    qkv[:, 0, 0] *= 2.0  # a sharper head
+    qkv_bits = synth.f32_to_bf16_bits(qkv)
+    w = synth.make_layer_weights(synth.rng(2), D=H * 64, H=H)
+    modes = np.zeros(H, np.int32)
+    modes[0] = 2
+    q = oracle.bf16_bits_to_f64(qkv_bits[:, :, 0].reshape(N, 3, 64))
+    mean_v = np.zeros((H, 64))
+    got = _run_heads(qkv_bits, w, N, H, modes, np.zeros((H, 64)), mean_v)
+    tail0 = 304 * 384  # first row of the last round's groups on 152 SMs (304 whole groups)
+    rows = np.unique(np.concatenate([np.arange(0, 64), np.arange(tail0 - 64, tail0 + 64),
+                                     np.arange(N - 64, N),
+                                     np.random.default_rng(1).choice(N, 256, replace=False)]))
+    want = oracle.full_attention(q[:, 0], q[:, 1], q[:, 2], rows=rows)
+    compare(got[rows, 0], oracle.round_bf16(want), what="full head, N = 137,400")
