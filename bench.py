@@ -504,7 +504,7 @@ def kernel_case(args):
     dev = torch.device("cuda:0")
     N = args.case_tokens
     qkv = torch.randn(N, 3 * D, device=dev).to(torch.bfloat16)
-    if args.kernel_case in ("layer_norm", "router", "surrogate"):
+    if args.kernel_case in ("layer_norm", "router", "surrogate", "mean"):
         w = vpb.to_device(synth.make_layer_weights(synth.rng(0), block=True), dev)
         dm = vpb.dims(N, H)
         ws = vpb.workspace(dm, vpb.VP_WS_ROUTER, dev)
@@ -515,7 +515,9 @@ def kernel_case(args):
         ctx = torch.zeros(H, d, device=dev)
         mv = torch.zeros(H, d, device=dev)
         ids = torch.arange(H, dtype=torch.int32, device=dev)
-        off = torch.tensor([0, 0, H, H], dtype=torch.int32, device=dev)
+        # all heads in one cheap mode: surrogate (offsets 0, 0, H, H) or mean (0, H, H, H)
+        off = torch.tensor([0, H, H, H] if args.kernel_case == "mean" else [0, 0, H, H], dtype=torch.int32,
+                           device=dev)
         for _ in range(args.case_launches):
             if args.kernel_case == "layer_norm":
                 vpb.vp_layer_norm(x, w["ln1_g"], w["ln1_b"], 1e-6, out=y)
@@ -523,6 +525,15 @@ def kernel_case(args):
                 vpb.vp_router(dm, qkv, vpb.router_weights(w), None, s, modes, None, ctx, mv, None, ws)
             else:
                 vpb.vp_head_attention(dm, qkv, ids, off, ctx, mv, vpb.surrogate_weights(w), y, ws)
+    elif args.kernel_case == "bin":
+        modes = torch.tensor([i % 3 for i in range(H)], dtype=torch.int32, device=dev)
+        ids = torch.empty(H, dtype=torch.int32, device=dev)
+        off = torch.empty(4, dtype=torch.int32, device=dev)
+        n_tiles = -(-N // 128)
+        work = torch.empty(H * n_tiles, 2, dtype=torch.int32, device=dev)
+        nw = torch.empty(1, dtype=torch.int32, device=dev)
+        for _ in range(args.case_launches):
+            vpb.vp_bin_heads(H, N, modes, ids, off, work, nw)
     elif args.kernel_case == "attn_full":
         w = vpb.to_device(synth.make_layer_weights(synth.rng(0)), dev)
         y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
@@ -574,7 +585,8 @@ def main():
     ap.add_argument("--no-s32", dest="s32", action="store_false")
     ap.add_argument("--variants", action="store_true", default=True)
     ap.add_argument("--no-variants", dest="variants", action="store_false")
-    ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "layer_norm", "router", "surrogate"],
+    ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "layer_norm", "router", "surrogate", "mean",
+                                              "bin"],
                     default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
     ap.add_argument("--case-tokens", type=int, default=32768)
