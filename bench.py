@@ -544,6 +544,21 @@ def kernel_case(args):
         z = torch.zeros(H, d, device=dev)
         for _ in range(args.case_launches):
             vpb.vp_head_attention(dm, qkv, ids, off, z, z, vpb.surrogate_weights(w), y, ws)
+    elif args.kernel_case == "gemm_fc1":  # FFN up-projection with the GELU epilogue
+        x = torch.randn(N, D, device=dev).to(torch.bfloat16)
+        w1 = (torch.rand(4 * D, D, device=dev) * 0.1 - 0.05).to(torch.bfloat16)
+        b1 = torch.randn(4 * D, device=dev) * 0.1
+        hid = torch.empty(N, 4 * D, dtype=torch.bfloat16, device=dev)
+        for _ in range(args.case_launches):
+            vpb.vp_linear(x, w1, b1, act=vpb.VP_ACT_GELU, out=hid)
+    elif args.kernel_case == "gemm_wo":  # W_O with bias, LayerScale and residual in place
+        x = torch.randn(N, D, device=dev).to(torch.bfloat16)
+        res = torch.randn(N, D, device=dev).to(torch.bfloat16)
+        wo = (torch.rand(D, D, device=dev) * 0.1 - 0.05).to(torch.bfloat16)
+        bo = torch.randn(D, device=dev) * 0.1
+        ls = torch.full((D,), 0.5, device=dev)
+        for _ in range(args.case_launches):
+            vpb.vp_linear(x, wo, bo, scale=ls, residual=res, out=res)
     else:
         x = torch.randn(N, D, device=dev).to(torch.bfloat16)
         wq = (torch.rand(3 * D, D, device=dev) * 0.1 - 0.05).to(torch.bfloat16)
@@ -585,8 +600,8 @@ def main():
     ap.add_argument("--no-s32", dest="s32", action="store_false")
     ap.add_argument("--variants", action="store_true", default=True)
     ap.add_argument("--no-variants", dest="variants", action="store_false")
-    ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "layer_norm", "router", "surrogate", "mean",
-                                              "bin"],
+    ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
+                                              "surrogate", "mean", "bin"],
                     default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
     ap.add_argument("--case-tokens", type=int, default=32768)

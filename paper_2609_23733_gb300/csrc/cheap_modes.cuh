@@ -224,8 +224,10 @@ __device__ __forceinline__ void surrogate_rows(const HeadAttnArgs& a, const Surr
     }
     const int col = 8 * j + 2 * c;
     const float c0 = sm.c1[col], c1v = sm.c1[col + 1];
-    hid[j][0] = pack_bf16x2(gelu_as(acc[0] + c0), gelu_as(acc[1] + c1v));
-    hid[j][1] = pack_bf16x2(gelu_as(acc[2] + c0), gelu_as(acc[3] + c1v));
+    const float2 ga = gelu_as2(fadd2(make_float2(acc[0], acc[1]), make_float2(c0, c1v)));
+    const float2 gb = gelu_as2(fadd2(make_float2(acc[2], acc[3]), make_float2(c0, c1v)));
+    hid[j][0] = pack_bf16x2(ga.x, ga.y);
+    hid[j][1] = pack_bf16x2(gb.x, gb.y);
   }
   // Layer 2: the accumulator layout of two adjacent n-tiles is the A-fragment layout of one
   // 16-wide k-step.  Output n-tile j of both MLPs is finished and stored before the next.

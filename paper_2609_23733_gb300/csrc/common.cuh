@@ -278,6 +278,16 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
   return d;
 }
 
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
 __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   float2 d;
   asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
@@ -329,6 +339,30 @@ __device__ __forceinline__ float erf_as(float x) {
 // GELU, erf form: 0.5 x (1 + erf(x / sqrt 2)).
 __device__ __forceinline__ float gelu_as(float x) {
   return 0.5f * x * (1.f + erf_as(x * 0.70710678118654752f));
+}
+
+// The same GELU for two values with packed f32x2 arithmetic.  With z = x / sqrt 2 and
+// erf(z) = sign(z) (1 - poly(t) e^{-z^2}) from 7.1.26, x (1 + erf(z)) = x + |x| r with
+// r = 1 - poly(t) e^{-z^2}, so no sign transfer is needed: gelu = 0.5 (x + |x| r).  The
+// polynomial is evaluated with negated coefficients, so that r = 1 + poly'(t) e^{-z^2}.
+__device__ __forceinline__ float2 gelu_as2(float2 x) {
+  const float kP = 0.3275911f * 0.70710678118654752f;  // p / sqrt 2: t = 1 / (1 + p |z|)
+  const float kE = -0.5f * 1.4426950408889634f;        // e^{-z^2} = 2^{kE x^2}
+  const float2 ax = make_float2(fabsf(x.x), fabsf(x.y));
+  const float2 d = ffma2(ax, make_float2(kP, kP), make_float2(1.f, 1.f));
+  float2 t;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t.x) : "f"(d.x));
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t.y) : "f"(d.y));
+  float2 p = ffma2(t, make_float2(-1.061405429f, -1.061405429f),
+                   make_float2(1.453152027f, 1.453152027f));
+  p = ffma2(t, p, make_float2(-1.421413741f, -1.421413741f));
+  p = ffma2(t, p, make_float2(0.284496736f, 0.284496736f));
+  p = ffma2(t, p, make_float2(-0.254829592f, -0.254829592f));
+  p = fmul2(p, t);
+  const float2 q = fmul2(ax, fmul2(ax, make_float2(kE, kE)));
+  const float2 e = make_float2(fast_exp2(q.x), fast_exp2(q.y));
+  const float2 r = ffma2(p, e, make_float2(1.f, 1.f));
+  return fmul2(ffma2(ax, r, x), make_float2(0.5f, 0.5f));
 }
 
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }

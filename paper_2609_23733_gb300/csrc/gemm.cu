@@ -160,6 +160,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
       const int mt = t / n_tiles, nt = t - mt * n_tiles;
       const uint32_t ab = i & 1;
+      if (prm.residual) {
+        // Pull this thread's residual row segment (128 columns, 256 bytes) into L2 while the
+        // tile's MMAs still run: read later from HBM, it would hold up the epilogue.
+        const int prow = mt * kBM + quarter * 32 + lane, pcol = nt * kBN + half * 128;
+        if (prow < M && pcol < N) {
+          const __nv_bfloat16* pp = prm.residual + (size_t)prow * N + pcol;
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(pp));
+          if (pcol + 64 < N) asm volatile("prefetch.global.L2 [%0];" ::"l"(pp + 64));
+        }
+      }
       const bool ok = mbar_wait_warp(&sm.acc_full[ab], (i >> 1) & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
@@ -176,21 +186,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         float* x = v[cc & 1];
         const int col0 = nt * kBN + half * 128 + cc * 32;
         if (col0 < N) {
+          // Bias, GELU, LayerScale and residual on column pairs (packed f32x2 arithmetic).
           if (prm.bias) {
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
               const float4 b4 = col0 + 4 * q + 3 < N
                                     ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-              x[4 * q] += b4.x;
-              x[4 * q + 1] += b4.y;
-              x[4 * q + 2] += b4.z;
-              x[4 * q + 3] += b4.w;
+              const float2 a0 = fadd2(make_float2(x[4 * q], x[4 * q + 1]), make_float2(b4.x, b4.y));
+              const float2 a1 = fadd2(make_float2(x[4 * q + 2], x[4 * q + 3]), make_float2(b4.z, b4.w));
+              x[4 * q] = a0.x;
+              x[4 * q + 1] = a0.y;
+              x[4 * q + 2] = a1.x;
+              x[4 * q + 3] = a1.y;
             }
           }
           if (prm.act == VP_ACT_GELU) {
 #pragma unroll
-            for (int k = 0; k < 32; ++k) x[k] = gelu_as(x[k]);
+            for (int k = 0; k < 16; ++k) {
+              const float2 gk = gelu_as2(make_float2(x[2 * k], x[2 * k + 1]));
+              x[2 * k] = gk.x;
+              x[2 * k + 1] = gk.y;
+            }
           }
           if (prm.scale) {
 #pragma unroll
@@ -198,10 +215,12 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float4 s4 = col0 + 4 * q + 3 < N
                                     ? __ldg(reinterpret_cast<const float4*>(prm.scale + col0) + q)
                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-              x[4 * q] *= s4.x;
-              x[4 * q + 1] *= s4.y;
-              x[4 * q + 2] *= s4.z;
-              x[4 * q + 3] *= s4.w;
+              const float2 a0 = fmul2(make_float2(x[4 * q], x[4 * q + 1]), make_float2(s4.x, s4.y));
+              const float2 a1 = fmul2(make_float2(x[4 * q + 2], x[4 * q + 3]), make_float2(s4.z, s4.w));
+              x[4 * q] = a0.x;
+              x[4 * q + 1] = a0.y;
+              x[4 * q + 2] = a1.x;
+              x[4 * q + 3] = a1.y;
             }
           }
           if (prm.residual && row_ok) {
@@ -213,8 +232,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t uw[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
-                  x[8 * q + 2 * k] += bf16_lo(uw[k]);
-                  x[8 * q + 2 * k + 1] += bf16_hi(uw[k]);
+                  const float2 a = fadd2(make_float2(x[8 * q + 2 * k], x[8 * q + 2 * k + 1]),
+                                         make_float2(bf16_lo(uw[k]), bf16_hi(uw[k])));
+                  x[8 * q + 2 * k] = a.x;
+                  x[8 * q + 2 * k + 1] = a.y;
                 }
               }
             }

@@ -28,3 +28,28 @@ def test_gelu_from_7_1_26_matches_exact_gelu():
     g = 0.5 * x * (1.0 + erf_as(x / np.sqrt(2.0)))
     exact = 0.5 * x * (1.0 + scipy.special.erf(x / np.sqrt(2.0)))
     assert np.max(np.abs(g - exact)) <= 1.5e-7 * 0.5 * 10
+
+
+def test_packed_gelu_form_matches_exact_gelu():
+    """The packed-pair GELU of the GEMM epilogue and the surrogate heads rewrites
+    x (1 + erf(x / sqrt 2)) as x + |x| r with r = 1 - poly(t) e^{-x^2 / 2} (7.1.26, t = 1 /
+    (1 + p |x| / sqrt 2)), evaluates poly with negated coefficients and forms e^{-x^2/2} as
+    2^(-log2(e) / 2 x^2); simulated here step by step in float32."""
+    f = np.float32
+    x = np.linspace(-10, 10, 200001).astype(f)
+    ax = np.abs(x)
+    d = (ax * f(P * 0.70710678118654752) + f(1)).astype(f)
+    t = (f(1) / d).astype(f)
+    p = (t * f(-A[4]) + f(-A[3])).astype(f)
+    p = (t * p + f(-A[2])).astype(f)
+    p = (t * p + f(-A[1])).astype(f)
+    p = (t * p + f(-A[0])).astype(f)
+    p = (p * t).astype(f)
+    q = (ax * (ax * f(-0.5 * 1.4426950408889634))).astype(f)
+    e = np.exp2(q.astype(np.float64)).astype(f)
+    r = (p * e + f(1)).astype(f)
+    g = ((ax * r + x) * f(0.5)).astype(np.float64)
+    xd = x.astype(np.float64)
+    exact = 0.5 * xd * (1.0 + scipy.special.erf(xd / np.sqrt(2.0)))
+    # float32 evaluation adds a few ulps of |x| to the formula's own 1.5e-7 bound
+    assert np.all(np.abs(g - exact) <= 1.5e-7 * 0.5 * np.abs(xd) + 4e-7 * np.abs(xd) + 1e-12)
