@@ -330,18 +330,20 @@ def run_ours(args):
         per_launch_flops = full_flops * args.steps / per_class_n["attn_full"]
         per_launch_ms = per_class_ms["attn_full"] / per_class_n["attn_full"]
         ach = per_launch_flops / (per_launch_ms * 1e-3) / 1e12
-        peak = pk.get("bf16_tflops_sustained") or 1700.0
+        peak = pk.get("bf16_tflops_sustained") or 1700.0  # fallback: an earlier GB300 measurement
         roof = {"bound": "tensor", "kernel": "attn_full_kernel", "achieved": ach, "peak": peak,
-                "unit": "TFLOP/s", "frac": ach / peak, "peak_kind": "measured sustained bf16 (cuBLAS)",
+                "unit": "TFLOP/s", "frac": ach / peak, "peak_kind": ("measured sustained bf16 (cuBLAS)" if pk.get("bf16_tflops_sustained")
+                                                                  else "fallback sustained bf16"),
                 "traffic": traffic_from_profile("attn_full"), "ms_per_launch": per_launch_ms,
                 "flop_per_launch": per_launch_flops}
     elif dominant == "gemm" and per_class_n["gemm"]:
         per_launch_flops = lin_flops * args.steps / per_class_n["gemm"]
         per_launch_ms = per_class_ms["gemm"] / per_class_n["gemm"]
         ach = per_launch_flops / (per_launch_ms * 1e-3) / 1e12
-        peak = pk.get("bf16_tflops_sustained") or 1700.0
+        peak = pk.get("bf16_tflops_sustained") or 1700.0  # fallback: an earlier GB300 measurement
         roof = {"bound": "tensor", "kernel": "gemm_kernel", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
-                "frac": ach / peak, "peak_kind": "measured sustained bf16 (cuBLAS)",
+                "frac": ach / peak, "peak_kind": ("measured sustained bf16 (cuBLAS)" if pk.get("bf16_tflops_sustained")
+                                                                  else "fallback sustained bf16"),
                 "traffic": traffic_from_profile("gemm"), "ms_per_launch": per_launch_ms}
 
     cpu = None
@@ -433,7 +435,7 @@ def variant_probe(vpb, dev, N, dw, pk):
     ctx = torch.randn(H, d, device=dev) * 0.1
     mv = torch.randn(H, d, device=dev) * 0.1
     sw = vpb.surrogate_weights(dw)
-    hbm = pk.get("hbm_gbs") or 6784.8
+    hbm = pk.get("hbm_gbs") or 6800.0  # fallback: an earlier GB300 measurement
     out = {}
     cases = [("surrogate", 0, [0, 0, H, H], 256), ("surrogate_no_residual", 4, [0, 0, H, H], 128),
              ("linear_attention", 8, [0, 0, H, H], 512), ("mean", 0, [0, H, H, H], 128)]
@@ -489,8 +491,9 @@ def full_attention_probe(vpb, dev, N, dw, pk):
     ms_sal = timed(s_attn)  # with the MaxAttn saliency epilogue (exact s_h^attn of every head)
     sal = s_attn.cpu().numpy()
     tf = 4.0 * N * N * d * H / (ms * 1e-3) / 1e12
-    peak = pk.get("bf16_tflops") or 1886.0
-    return {"ms": ms, "tflops": tf, "peak": peak, "frac": tf / peak, "peak_kind": "measured burst bf16",
+    peak = pk.get("bf16_tflops") or 1900.0  # fallback: an earlier GB300 measurement
+    return {"ms": ms, "tflops": tf, "peak": peak, "frac": tf / peak,
+            "peak_kind": "measured burst bf16" if pk.get("bf16_tflops") else "fallback burst bf16",
             "max_attn_saliency": {"ms": ms_sal, "min": float(sal.min()), "max": float(sal.max()),
                                   "note": "same launch with the exact s_h^attn = max_ij A_ij output on"}}
 
