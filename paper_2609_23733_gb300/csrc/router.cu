@@ -34,16 +34,23 @@ __device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, uint
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-// tanh(x) * sigma(y) = (1 - e^-2x) / ((1 + e^-2x)(1 + e^-y)).  Arguments are clamped so
-// that the product of the two exponentials stays finite in fp32 (|x| <= 20 leaves tanh
-// at +-1 to fp32 precision; sigma(-40) < 5e-18).
-__device__ __forceinline__ float tanh_times_sigmoid(float x, float y) {
+// tanh(x) * sigma(y) for the pooling logits of §4.1, two at a time on packed f32x2 pairs, in a
+// form that needs no clamps:
+// tanh(x) = sign(x) (1 - e^{-2|x|}) / (1 + e^{-2|x|}) with e^{-2|x|} <= 1, and
+// sigma(y) = 1 / (1 + e^{-y}), whose e^{-y} may overflow to +inf, giving 0 as it should.
+__device__ __forceinline__ float2 tanh_times_sigmoid2(float2 x, float2 y) {
   const float kLog2e = 1.4426950408889634f;
-  x = fminf(fmaxf(x, -20.f), 20.f);
-  y = fminf(fmaxf(y, -40.f), 40.f);
-  const float ea = fast_exp2(-2.f * kLog2e * x);
-  const float eb = fast_exp2(-kLog2e * y);
-  return __fdividef(1.f - ea, (1.f + ea) * (1.f + eb));
+  const float2 a = fmul2(make_float2(fabsf(x.x), fabsf(x.y)), make_float2(-2.f * kLog2e, -2.f * kLog2e));
+  const float2 b = fmul2(y, make_float2(-kLog2e, -kLog2e));
+  const float2 ea = make_float2(fast_exp2(a.x), fast_exp2(a.y));
+  const float2 eb = make_float2(fast_exp2(b.x), fast_exp2(b.y));
+  const float2 num = ffma2(ea, make_float2(-1.f, -1.f), make_float2(1.f, 1.f));
+  const float2 den = fmul2(fadd2(ea, make_float2(1.f, 1.f)), fadd2(eb, make_float2(1.f, 1.f)));
+  float2 r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r.x) : "f"(den.x));
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r.y) : "f"(den.y));
+  const float2 t = fmul2(num, r);
+  return make_float2(copysignf(t.x, x.x), copysignf(t.y, x.y));
 }
 
 __device__ __forceinline__ void token_range(int N, int n_split, int split, int align, int& t0,
@@ -63,8 +70,8 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
   const bool mean_pool = (a.variant & VP_VARIANT_MEAN_QPOOL) != 0;  // §5 component ablation
 
   __shared__ __align__(16) __nv_bfloat16 sB[128 * kBStride];  // rows 0..63 W_h, 64..127 U_h
-  __shared__ float s_bias[128];                              // bW | bU
-  __shared__ float s_w[64];
+  __shared__ __align__(16) float s_bias[128];                // bW | bU
+  __shared__ __align__(16) float s_w[64];
   __shared__ float s_part[4][kPoolPartial];
 
   const int tid = threadIdx.x;
@@ -126,16 +133,22 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
       }
     }
     // Pooling logits: columns 8j + 2c + e of the W half (j < 8) pair with the same
-    // columns of the U half (j + 8) in the same thread.
+    // columns of the U half (j + 8) in the same thread; the two columns e = 0, 1 of a row
+    // form one packed pair.
+    float2 pa = make_float2(0.f, 0.f), pb = make_float2(0.f, 0.f);
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int l = 8 * j + 2 * c + e;
-        ea += s_w[l] * tanh_times_sigmoid(acc[j][e] + s_bias[l], acc[j + 8][e] + s_bias[64 + l]);
-        eb += s_w[l] * tanh_times_sigmoid(acc[j][2 + e] + s_bias[l], acc[j + 8][2 + e] + s_bias[64 + l]);
-      }
+      const int l = 8 * j + 2 * c;
+      const float2 bw = *reinterpret_cast<const float2*>(&s_bias[l]);
+      const float2 bu = *reinterpret_cast<const float2*>(&s_bias[64 + l]);
+      const float2 wl = *reinterpret_cast<const float2*>(&s_w[l]);
+      pa = ffma2(wl, tanh_times_sigmoid2(fadd2(make_float2(acc[j][0], acc[j][1]), bw),
+                                         fadd2(make_float2(acc[j + 8][0], acc[j + 8][1]), bu)), pa);
+      pb = ffma2(wl, tanh_times_sigmoid2(fadd2(make_float2(acc[j][2], acc[j][3]), bw),
+                                         fadd2(make_float2(acc[j + 8][2], acc[j + 8][3]), bu)), pb);
     }
+    ea = pa.x + pa.y;
+    eb = pb.x + pb.y;
     ea += __shfl_xor_sync(0xffffffffu, ea, 1);
     ea += __shfl_xor_sync(0xffffffffu, ea, 2);
     eb += __shfl_xor_sync(0xffffffffu, eb, 1);
@@ -349,7 +362,6 @@ __global__ void __launch_bounds__(kKeyThreads) router_keys_kernel(RouterArgs a, 
   if (!s_last) return;
   __threadfence();
   // Last CTA of head h: saliency, context, mean of V, mode.
-  __shared__ float s_L;
   if (tid < 64) {
     const float* pp = sc.key_part + (size_t)h * kKeySplitMax * kKeyPartial;
     float Mx = -INFINITY;
@@ -383,7 +395,6 @@ __global__ void __launch_bounds__(kKeyThreads) router_keys_kernel(RouterArgs a, 
       sc.key_stats[2 * h + 1] = ll;
       if (a.s_out) a.s_out[h] = s;
       if (a.modes_out) a.modes_out[h] = mode;
-      s_L = ll;
     }
   }
   // The last head to finish groups all heads by mode.
