@@ -99,18 +99,29 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
 #pragma unroll
   for (int i = 0; i < 16; ++i) accq[i] = 0.f;
 
+  // Each thread holds channels 16c..16c+15 of rows ra and rb.  The MMA's reduction index k
+  // is permuted consistently in A and B (logical k pair (kk, 2c) <-> channels 16c + 4kk +
+  // {0,1}, pair (kk, 2c + 8) <-> 16c + 4kk + {2,3}), so that every thread reads 32 contiguous
+  // bytes of its rows and of the weight rows.  The next tile's rows are loaded while the
+  // current tile is computed.
+  auto load_rows = [&](int base, uint4& x0, uint4& x1, uint4& y0, uint4& y1) {
+    const int ra = base + r, rb = base + r + 8;
+    const uint4* pa = reinterpret_cast<const uint4*>(qbase + (size_t)(ra < t1 ? ra : t0) * row_pitch);
+    const uint4* pb = reinterpret_cast<const uint4*>(qbase + (size_t)(rb < t1 ? rb : t0) * row_pitch);
+    x0 = __ldg(pa);
+    x1 = __ldg(pa + 1);
+    y0 = __ldg(pb);
+    y1 = __ldg(pb + 1);
+  };
+  uint4 nx0, nx1, ny0, ny1;
+  if (t0 + 16 * warp < t1) load_rows(t0 + 16 * warp, nx0, nx1, ny0, ny1);
   for (int base = t0 + 16 * warp; base < t1; base += 64) {
     const int ra = base + r, rb = base + r + 8;
     const bool va = ra < t1, vb = rb < t1;
-    // Each thread holds channels 16c..16c+15 of rows ra and rb.  The MMA's reduction
-    // index k is permuted consistently in A and B (logical k pair (kk, 2c) <-> channels
-    // 16c + 4kk + {0,1}, pair (kk, 2c + 8) <-> 16c + 4kk + {2,3}), so that every thread
-    // reads 32 contiguous bytes of its rows and of the weight rows.
     uint32_t qa[8], qb[8];
     {
-      const uint4* pa = reinterpret_cast<const uint4*>(qbase + (size_t)(va ? ra : t0) * row_pitch);
-      const uint4* pb = reinterpret_cast<const uint4*>(qbase + (size_t)(vb ? rb : t0) * row_pitch);
-      uint4 x0 = __ldg(pa), x1 = __ldg(pa + 1), y0 = __ldg(pb), y1 = __ldg(pb + 1);
+      const uint4 x0 = nx0, x1 = nx1, y0 = ny0, y1 = ny1;
+      if (base + 64 < t1) load_rows(base + 64, nx0, nx1, ny0, ny1);
       qa[0] = x0.x; qa[1] = x0.y; qa[2] = x0.z; qa[3] = x0.w;
       qa[4] = x1.x; qa[5] = x1.y; qa[6] = x1.z; qa[7] = x1.w;
       qb[0] = y0.x; qb[1] = y0.y; qb[2] = y0.z; qb[3] = y0.w;
@@ -281,17 +292,28 @@ __global__ void __launch_bounds__(kKeyThreads) router_keys_kernel(RouterArgs a, 
   // The loop bound is uniform across the CTA so that the 8-lane shuffles below always
   // run with the whole warp; rows past t1 are loaded from row t0 and masked.  Four rows per
   // row group are in flight (eight 16-byte loads per thread) before any arithmetic.
+  // The next batch of rows is loaded while the current one is computed.
+  uint4 nk[4], nv[4];
+  auto load_batch = [&](int base) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int row = base + g + 32 * u;
+      const size_t o = (size_t)(row < t1 ? row : t0) * row_pitch;
+      nk[u] = __ldg(reinterpret_cast<const uint4*>(kb + o));
+      nv[u] = __ldg(reinterpret_cast<const uint4*>(vb + o));
+    }
+  };
+  if (t0 < t1) load_batch(t0);
   for (int base = t0; base < t1; base += 128) {
     uint4 kr[4], vr[4];
     bool valid[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const int row = base + g + 32 * u;
-      valid[u] = row < t1;
-      const size_t o = (size_t)(valid[u] ? row : t0) * row_pitch;
-      kr[u] = __ldg(reinterpret_cast<const uint4*>(kb + o));
-      vr[u] = __ldg(reinterpret_cast<const uint4*>(vb + o));
+      kr[u] = nk[u];
+      vr[u] = nv[u];
+      valid[u] = base + g + 32 * u < t1;
     }
+    if (base + 128 < t1) load_batch(base + 128);
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const uint32_t kw[4] = {kr[u].x, kr[u].y, kr[u].z, kr[u].w};
