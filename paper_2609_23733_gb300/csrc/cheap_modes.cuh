@@ -34,7 +34,17 @@ __device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, uint
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ float sigmoidf(float x) { return 1.f / (1.f + __expf(-x)); }
+// sigma(x) = 1 / (1 + e^{-x}) for a packed pair (MUFU ex2 and approximate reciprocal; an
+// overflowing e^{-x} gives 0).
+__device__ __forceinline__ float2 sigmoid2(float2 x) {
+  const float kLog2e = 1.4426950408889634f;
+  const float2 a = fmul2(x, make_float2(-kLog2e, -kLog2e));
+  const float2 d = make_float2(1.f + fast_exp2(a.x), 1.f + fast_exp2(a.y));
+  float2 r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r.x) : "f"(d.x));
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r.y) : "f"(d.y));
+  return r;
+}
 
 struct SurrSmem {
   __nv_bfloat16 w1[128 * kBStride];  // rows 0..63: MLP_gamma layer 1 (value half), 64..127: MLP_delta
@@ -251,15 +261,15 @@ __device__ __forceinline__ void surrogate_rows(const HeadAttnArgs& a, const Surr
     }
     // y = C + sigma(gamma) (.) delta, stored as bf16 in Y[row][h][:].
     const int col = 8 * j + 2 * c;
-    const float C0 = sm.ctx[col], C1 = sm.ctx[col + 1];
-    const float bg0 = sm.b2[col], bg1 = sm.b2[col + 1];
-    const float bd0 = sm.b2[64 + col], bd1 = sm.b2[64 + col + 1];
-    if (va)
-      *reinterpret_cast<uint32_t*>(ya + col) =
-          pack_bf16x2(C0 + sigmoidf(og[0] + bg0) * (od[0] + bd0), C1 + sigmoidf(og[1] + bg1) * (od[1] + bd1));
-    if (vb)
-      *reinterpret_cast<uint32_t*>(yb + col) =
-          pack_bf16x2(C0 + sigmoidf(og[2] + bg0) * (od[2] + bd0), C1 + sigmoidf(og[3] + bg1) * (od[3] + bd1));
+    const float2 C = *reinterpret_cast<const float2*>(&sm.ctx[col]);
+    const float2 bg = *reinterpret_cast<const float2*>(&sm.b2[col]);
+    const float2 bd = *reinterpret_cast<const float2*>(&sm.b2[64 + col]);
+    const float2 ya2 = ffma2(sigmoid2(fadd2(make_float2(og[0], og[1]), bg)),
+                             fadd2(make_float2(od[0], od[1]), bd), C);
+    const float2 yb2 = ffma2(sigmoid2(fadd2(make_float2(og[2], og[3]), bg)),
+                             fadd2(make_float2(od[2], od[3]), bd), C);
+    if (va) *reinterpret_cast<uint32_t*>(ya + col) = pack_bf16x2(ya2.x, ya2.y);
+    if (vb) *reinterpret_cast<uint32_t*>(yb + col) = pack_bf16x2(yb2.x, yb2.y);
   }
 }
 
