@@ -118,10 +118,14 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
 
     (1) X~ = LN1(X); (2) routed attention -> Y; (3) A = LS1(Y W_O),
     X_attn = X + A; (4) Z~ = LN2(X_attn), F = LS2(FFN(Z~)), X' = X_attn + F.
-    FFN = Linear(D -> 4D) -> GELU -> Linear(4D -> D).  Returns (X', info)."""
+    FFN = Linear(D -> 4D) -> GELU -> Linear(4D -> D).  Returns (X', info).
+
+    Storage points (materialize, bf16): QKV, Y, Z~, the FFN hidden layer and the residual
+    stream X_attn, X'.  The LN1 output X~ is not stored: the block feeds it straight into
+    the QKV projection."""
     mat = materialize or _identity
     X = np.asarray(X, np.float64)
-    Xt = mat(layer_norm(X, lw["ln1_g"], lw["ln1_b"], eps))
+    Xt = layer_norm(X, lw["ln1_g"], lw["ln1_b"], eps)
     att = moh_attention(Xt, lw, force_modes=force_modes, materialize=materialize,
                         tau_low=tau_low, tau_high=tau_high, variant=variant)
     A = (att["Y"] @ lw["w_o"].T + lw["b_o"]) * lw["ls1"]

@@ -154,10 +154,17 @@ size_t layer_ws_bytes(const vp_dims* dm) {
   return heads_scratch_bytes(dm->H) + align_up(N * 3 * D * 2) + align_up(N * D * 2);
 }
 
+// The stack's LayerNorm scratch: LN1's row statistics (per 128-column block), the current
+// block's folded QKV weights with their column sums and biases, and the LN2 output.
+size_t ln_scratch_bytes(size_t N, size_t D) {
+  return align_up(N * (D / 128) * sizeof(float2)) + align_up(3 * D * D * 2) +
+         2 * align_up(3 * D * sizeof(float)) + align_up(N * D * 2);
+}
+
 size_t stack_ws_bytes(const vp_dims* dm) {
   const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
-  // x~ (LN output) + one region shared by {QKV, Y} and the FFN hidden layer.
-  return heads_scratch_bytes(dm->H) + align_up(N * D * 2) + align_up(N * 4 * D * 2);
+  // LayerNorm scratch + one region shared by {QKV, Y} and the FFN hidden layer.
+  return heads_scratch_bytes(dm->H) + ln_scratch_bytes(N, D) + align_up(N * 4 * D * 2);
 }
 
 // Row widths the LayerNorm kernel is instantiated for.
@@ -248,13 +255,21 @@ vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* 
 }
 
 // QKV projection -> router -> bins -> heads -> W_O (+ optional LayerScale / residual).
+// LayerNorm folded into a layer's QKV projection: xin is then the raw residual stream and
+// w_qkv / b_qkv the folded weights (see LinearArgs).
+struct LnFold {
+  const float2* part_in;
+  const float* c;
+  float eps;
+};
+
 vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* w_qkv,
                     const float* b_qkv, const vp_bf16* w_o, const float* b_o, const float* ls1,
                     const __nv_bfloat16* residual, const vp_router_weights* rw,
                     const vp_surrogate_weights* sw, const int32_t* force_modes,
                     __nv_bfloat16* out, __nv_bfloat16* qkv, __nv_bfloat16* y, float* s_out,
                     float* s_attn_out, int32_t* modes_out, const RouterScratch& sc,
-                    cudaStream_t st) {
+                    cudaStream_t st, const LnFold* fold = nullptr) {
   const int N = dm->N, D = dm->H * kHeadDim;
   const int sms = device_sm_count();
   LinearArgs la{};
@@ -267,6 +282,11 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
   la.act = VP_ACT_NONE;
   la.out = qkv;
   la.err = sc.err;
+  if (fold) {
+    la.ln_part = fold->part_in;
+    la.ln_c = fold->c;
+    la.ln_eps = fold->eps;
+  }
   VP_TRY(from_cuda(launch_linear(la, sms, st)));
   RouterArgs ra = make_router_args(dm, reinterpret_cast<const vp_bf16*>(qkv), rw, force_modes);
   ra.s_out = s_out;
@@ -527,30 +547,47 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
   const size_t N = dims->N;
   RouterScratch sc = carve_router_scratch(ws, dims->H);
   char* p = static_cast<char*>(ws) + heads_scratch_bytes(dims->H);
-  __nv_bfloat16* xt = reinterpret_cast<__nv_bfloat16*>(p);
+  // LayerNorm scratch (see ln_scratch_bytes).  LN1 is folded into the QKV projection, which
+  // then reads the raw residual stream; its row statistics come from the kernel that last
+  // wrote the stream (the previous block's FFN-down, or a statistics pass for the first
+  // block).  LN2 stays a kernel of its own: folded into the FFN-up projection it costs that
+  // GEMM's GELU epilogue more than the LayerNorm pass it saves.
+  float2* part = reinterpret_cast<float2*>(p);  // LN1 input statistics
+  p += align_up(N * (D / 128) * sizeof(float2));
+  __nv_bfloat16* wq = reinterpret_cast<__nv_bfloat16*>(p);  // [3D][D] folded W_qkv
+  p += align_up((size_t)3 * D * D * 2);
+  float* cq = reinterpret_cast<float*>(p);
+  p += align_up((size_t)3 * D * sizeof(float));
+  float* bq = reinterpret_cast<float*>(p);
+  p += align_up((size_t)3 * D * sizeof(float));
+  __nv_bfloat16* zt = reinterpret_cast<__nv_bfloat16*>(p);  // LN2 output
   p += align_up(N * D * 2);
   __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
   __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p + align_up(N * 3 * D * 2));
   __nv_bfloat16* hid = reinterpret_cast<__nv_bfloat16*>(p);  // reuses the QKV / Y region
   __nv_bfloat16* x = reinterpret_cast<__nv_bfloat16*>(x_inout);
   const int sms = device_sm_count();
+  VP_TRY(from_cuda(launch_ln_partials(dims->N, D, x, part, st)));
   for (int l = 0; l < n_layers; ++l) {
     const vp_layer_weights& w = layers[l];
-    // (1) X~ = LN1(X)
-    VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln1_g, w.ln1_b, ln_eps, xt, st)));
-    // (2)-(3) routed attention; X <- X + LS1 (Y W_O + b_O) in place
-    VP_TRY(run_layer(dims, xt, w.w_qkv, w.b_qkv, w.w_o, w.b_o, w.ls1, x, &w.router, &w.surrogate,
+    VP_TRY(from_cuda(launch_ln_fold_weights(3 * D, D,
+                                            reinterpret_cast<const __nv_bfloat16*>(w.w_qkv),
+                                            w.ln1_g, w.ln1_b, w.b_qkv, wq, cq, bq, st)));
+    // (1)-(3) X <- X + LS1 (Y W_O + b_O) in place, Y the routed attention of LN1(X)
+    const LnFold fold{part, cq, ln_eps};
+    VP_TRY(run_layer(dims, x, reinterpret_cast<const vp_bf16*>(wq), bq, w.w_o, w.b_o, w.ls1, x,
+                     &w.router, &w.surrogate,
                      force_modes ? force_modes + (size_t)l * dims->H : nullptr, x, qkv, y,
                      s_out ? s_out + (size_t)l * dims->H : nullptr,
                      s_attn_out ? s_attn_out + (size_t)l * dims->H : nullptr,
-                     modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st));
+                     modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st, &fold));
     // (4) Z~ = LN2(X_attn); X <- X_attn + LS2 FFN(Z~)
-    VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, xt, st)));
+    VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, zt, st)));
     LinearArgs f1{};
     f1.M = dims->N;
     f1.N = 4 * D;
     f1.K = D;
-    f1.A = xt;
+    f1.A = zt;
     f1.W = reinterpret_cast<const __nv_bfloat16*>(w.w_fc1);
     f1.bias = w.b_fc1;
     f1.act = VP_ACT_GELU;
@@ -569,6 +606,7 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     f2.residual = x;
     f2.out = x;
     f2.err = sc.err;
+    f2.part_out = part;  // the next block's LN1 statistics
     VP_TRY(from_cuda(launch_linear(f2, sms, st)));
   }
   return VP_OK;

@@ -1,5 +1,7 @@
 // Dense projections of Algorithm 1 (QKV, W_O, FFN) on the sm_103a tensor cores:
 //   out[M][N] = residual + scale (.) act(A[M][K] W[N][K]^T + bias)
+// optionally with a LayerNorm of A's rows folded in (A W^T -> rstd (A W^T - mu c^T), see
+// LinearArgs) and with the output rows' LayerNorm statistics as (mean, M2) per 128 columns.
 // Persistent CTAs (one per SM), 128 x 256 output tiles, 64-wide K blocks through a 4-stage
 // TMA ring (128-byte swizzle), tcgen05.mma (M=128, N=256, K=16, bf16 -> fp32) into one of
 // two TMEM accumulators, so the epilogue of tile i overlaps the main loop of tile i+1.
@@ -43,6 +45,10 @@ struct GemmParams {
   const __nv_bfloat16* residual;
   __nv_bfloat16* out;
   unsigned int* err;
+  const float2* ln_part;
+  const float* ln_c;
+  float ln_eps;
+  float2* part_out;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -170,12 +176,50 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (pcol + 64 < N) asm volatile("prefetch.global.L2 [%0];" ::"l"(pp + 64));
         }
       }
-      const bool ok = mbar_wait_warp(&sm.acc_full[ab], (i >> 1) & 1, prm.err, abort_flag);
-      if (!ok) break;
-      tc_fence_after();
       const int row0 = mt * kBM + quarter * 32;
       const int row = row0 + lane;
       const bool row_ok = row < M;
+      // Folded LayerNorm: this row's mean and 1 / sqrt(var + eps) from the (mean, M2) of its
+      // 128-column blocks (equal counts: M2 = sum M2_b + 128 sum (mean_b - mean)^2).  The
+      // first eight blocks (K = 1,024) are loaded before the accumulator wait.
+      float ln_mu = 0.f, ln_rstd = 1.f;
+      float4 lnp[4];
+      const int nb = K >> 7;  // even (K % 256 == 0)
+      const float4* lpp = reinterpret_cast<const float4*>(prm.ln_part + (size_t)row * nb);
+      if (prm.ln_part && row_ok) {
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+          if (2 * b < nb) lnp[b] = __ldg(lpp + b);
+      }
+      const bool ok = mbar_wait_warp(&sm.acc_full[ab], (i >> 1) & 1, prm.err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      if (prm.ln_part && row_ok) {
+        float sm_ = 0.f;
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+          if (2 * b < nb) sm_ += lnp[b].x + lnp[b].z;
+        for (int b = 4; 2 * b < nb; ++b) {
+          const float4 p4 = __ldg(lpp + b);
+          sm_ += p4.x + p4.z;
+        }
+        ln_mu = sm_ / (float)nb;
+        float m2 = 0.f;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          if (2 * b < nb) {
+            const float d0 = lnp[b].x - ln_mu, d1 = lnp[b].z - ln_mu;
+            m2 += lnp[b].y + lnp[b].w + 128.f * (d0 * d0 + d1 * d1);
+          }
+        }
+        for (int b = 4; 2 * b < nb; ++b) {
+          const float4 p4 = __ldg(lpp + b);
+          const float d0 = p4.x - ln_mu, d1 = p4.z - ln_mu;
+          m2 += p4.y + p4.w + 128.f * (d0 * d0 + d1 * d1);
+        }
+        ln_rstd = rsqrtf(m2 / (float)K + prm.ln_eps);
+      }
+      float cmean[4], cm2[4];  // output statistics per 32-column chunk (part_out)
       const uint32_t tcol = t_lane + ab * kBN + half * 128;
       float v[2][32];
       tmem_ld32(tcol, v[0]);
@@ -187,7 +231,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int col0 = nt * kBN + half * 128 + cc * 32;
         if (col0 < N) {
           // Bias, GELU, LayerScale and residual on column pairs (packed f32x2 arithmetic).
-          if (prm.bias) {
+          if (prm.ln_part) {  // rstd (acc - mu c) + bias'
+            const float2 nmu = make_float2(-ln_mu, -ln_mu), rs = make_float2(ln_rstd, ln_rstd);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const bool in = col0 + 4 * q + 3 < N;
+              const float4 c4 = in ? __ldg(reinterpret_cast<const float4*>(prm.ln_c + col0) + q)
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+              const float4 b4 = in ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+              const float2 a0 = ffma2(rs, ffma2(nmu, make_float2(c4.x, c4.y),
+                                                make_float2(x[4 * q], x[4 * q + 1])),
+                                      make_float2(b4.x, b4.y));
+              const float2 a1 = ffma2(rs, ffma2(nmu, make_float2(c4.z, c4.w),
+                                                make_float2(x[4 * q + 2], x[4 * q + 3])),
+                                      make_float2(b4.z, b4.w));
+              x[4 * q] = a0.x;
+              x[4 * q + 1] = a0.y;
+              x[4 * q + 2] = a1.x;
+              x[4 * q + 3] = a1.y;
+            }
+          } else if (prm.bias) {
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
               const float4 b4 = col0 + 4 * q + 3 < N
@@ -240,6 +304,20 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
           }
+          if (prm.part_out) {  // chunk mean and M2 (two passes over registers)
+            float2 s2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < 16; ++k) s2 = fadd2(s2, make_float2(x[2 * k], x[2 * k + 1]));
+            const float cm = (s2.x + s2.y) * (1.f / 32.f);
+            float2 q2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+              const float2 dd = fadd2(make_float2(x[2 * k], x[2 * k + 1]), make_float2(-cm, -cm));
+              q2 = ffma2(dd, dd, q2);
+            }
+            cmean[cc] = cm;
+            cm2[cc] = q2.x + q2.y;
+          }
           // Stage the 32 x 32 block (row = lane, 64 bytes) in the 64-byte swizzle the
           // output tensor map uses: 16-byte chunk q of row r sits at chunk q ^ ((r >> 1) & 3).
           unsigned char* buf = stg + (nst & 1) * 2048;
@@ -269,6 +347,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive(&sm.acc_empty[ab]);
         }
       }
+      const int pcol = nt * kBN + half * 128;  // this thread's 128-column block
+      if (prm.part_out && row_ok && pcol < N) {
+        const float mb = 0.25f * (cmean[0] + cmean[1] + cmean[2] + cmean[3]);
+        float m2 = cm2[0] + cm2[1] + cm2[2] + cm2[3];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) m2 += 32.f * (cmean[k] - mb) * (cmean[k] - mb);
+        prm.part_out[(size_t)row * (N >> 7) + (pcol >> 7)] = make_float2(mb, m2);
+      }
     }
     if (elect_one()) tma_store_wait_all();
     __syncwarp();
@@ -296,7 +382,11 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int tiles = ((a.M + kBM - 1) / kBM) * ((a.N + kBN - 1) / kBN);
-  GemmParams prm{a.M, a.N, a.K, a.bias, a.act, a.scale, a.residual, a.out, a.err};
+  if ((a.ln_part && (a.K % 256 != 0 || !a.ln_c || !a.bias)) ||
+      (a.part_out && a.N % 128 != 0))
+    return cudaErrorInvalidValue;
+  GemmParams prm{a.M,     a.N,   a.K,   a.bias,      a.act,  a.scale,   a.residual,
+                 a.out,   a.err, a.ln_part, a.ln_c, a.ln_eps, a.part_out};
   prof_before(VP_KERNEL_GEMM, st);
   gemm_kernel<<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
   prof_after(st);

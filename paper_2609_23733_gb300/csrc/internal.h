@@ -127,8 +127,26 @@ struct LinearArgs {
   const __nv_bfloat16* residual;
   __nv_bfloat16* out;
   unsigned int* err;   // may be NULL (vp_linear has no workspace): a private word is used
+  // LayerNorm folded into the projection (A is the un-normalised residual stream): with
+  // W' = W diag(gamma), c = W' 1 and bias' = b + W beta prepared by launch_ln_fold_weights,
+  //   LN(A) W^T + b = rstd_r (A W'^T - mu_r c^T) + bias',
+  // mu_r, rstd_r combined from ln_part (K % 128 == 0).  ln_part NULL: no LayerNorm.
+  const float2* ln_part;  // [M][K / 128] (mean, M2) of the 128-column blocks of A's rows
+  const float* ln_c;      // [N] column sums of W'
+  float ln_eps;
+  float2* part_out;       // [M][N / 128] (mean, M2) blocks of the output rows, or NULL (N % 128 == 0)
 };
 cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st);
+
+// Per-row LayerNorm statistics as (mean, M2) of 128-column blocks: x [M][D] bf16 ->
+// part [M][D / 128] float2 (D % 256 == 0, D <= 4096).
+cudaError_t launch_ln_partials(int M, int D, const __nv_bfloat16* x, float2* part, cudaStream_t st);
+// The folded LayerNorm's weights for a projection W [Nout][K] (nn.Linear layout):
+// Wp = W diag(g) (bf16), c[o] = sum_k Wp[o][k] (of the bf16 Wp), bp[o] = b[o] + sum_k W[o][k] beta[k]
+// (b NULL: 0).  K % 256 == 0, K <= 4096.
+cudaError_t launch_ln_fold_weights(int Nout, int K, const __nv_bfloat16* W, const float* g,
+                                   const float* beta, const float* b, __nv_bfloat16* Wp,
+                                   float* c, float* bp, cudaStream_t st);
 
 cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float* g,
                               const float* b, float eps, __nv_bfloat16* out, cudaStream_t st);

@@ -51,7 +51,10 @@ def test_workspace_sizes(vp):
     r = vp.vp_workspace_size(small, vp.VP_WS_ROUTER)
     assert r == vp.vp_workspace_size(big, vp.VP_WS_ROUTER)  # router scratch is independent of N
     assert vp.vp_workspace_size(big, vp.VP_WS_LAYER) >= r + 137400 * 4 * 1024 * 2
-    assert vp.vp_workspace_size(big, vp.VP_WS_STACK) >= r + 137400 * 5 * 1024 * 2
+    # stack: {QKV, Y} / FFN hidden region, the LN2 output, LN1 row statistics (8 blocks of
+    # (mean, M2) per row) and one block's folded QKV weights
+    assert vp.vp_workspace_size(big, vp.VP_WS_STACK) >= (r + 137400 * 5 * 1024 * 2 + 137400 * 8 * 8
+                                                         + 3 * 1024 * 1024 * 2)
     with pytest.raises(vp.VPError) as e:
         vp.vp_workspace_size(vp.dims(100, d=32), vp.VP_WS_ROUTER)
     assert e.value.status == 2
