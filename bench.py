@@ -382,6 +382,8 @@ def run_ours(args):
         line["stack_s32"] = s32_probe(vpb, dev)
     if args.variants:
         line["cheap_mode_variants"] = variant_probe(vpb, dev, N, dws[0], pk)
+    if args.qk:
+        line["qkv_positional"] = qk_probe(vpb, dev, N, dws[0])
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
@@ -459,6 +461,39 @@ def variant_probe(vpb, dev, N, dw, pk):
         out[name] = {"ms_16_heads": ms, "gb_s": gbs, "hbm_frac": gbs / hbm}
     out["tokens"] = N
     return out
+
+
+def qk_probe(vpb, dev, N, dw):
+    """Cost of the QKV step's positional information (qk-norm + 2-D RoPE, the library's
+    reading of the undefined P) at the stack's size: one routed layer with every head forced
+    to mean, with and without the options, and the projections' profiled time (QKV + W_O)."""
+    import torch
+    views = N // synth.tokens_per_view(518)
+    x = torch.randn(N, D, device=dev).to(torch.bfloat16)
+    out = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_LAYER, dev)
+    fm = torch.zeros(H, dtype=torch.int32, device=dev)
+    q = vpb.to_device(synth.make_qk_norm_weights(synth.rng(7)), dev)
+    opts = vpb.qk_options(q, norm_eps=1e-6, rope=True, tokens_per_view=synth.tokens_per_view(518),
+                          patch_start=5, grid_w=518 // 14, rope_base=100.0)
+    res = {"tokens": N, "views": views}
+    for name, qk in (("plain", None), ("qk_norm_rope", opts)):
+        def run():
+            vpb.vp_moh_global_attention(dm, x, dw["w_qkv"], dw["b_qkv"], dw["w_o"], dw["b_o"],
+                                        vpb.router_weights(dw), vpb.surrogate_weights(dw), fm, out, None, None,
+                                        None, None, ws, qk=qk)
+        for _ in range(2):
+            run()
+        torch.cuda.synchronize()
+        vpb.vp_profile_begin(64 * 5)
+        for _ in range(5):
+            run()
+        torch.cuda.synchronize()
+        _, cnt, ms = vpb.vp_profile_end()
+        res[f"gemm_ms_{name}"] = ms["gemm"] / 5
+    res["qk_epilogue_ms"] = res["gemm_ms_qk_norm_rope"] - res["gemm_ms_plain"]
+    return res
 
 
 def full_attention_probe(vpb, dev, N, dw, pk):
@@ -603,6 +638,7 @@ def main():
     ap.add_argument("--no-s32", dest="s32", action="store_false")
     ap.add_argument("--variants", action="store_true", default=True)
     ap.add_argument("--no-variants", dest="variants", action="store_false")
+    ap.add_argument("--no-qk", dest="qk", action="store_false")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
                                               "surrogate", "mean", "bin"],
                     default=None,

@@ -109,6 +109,33 @@ typedef struct vp_surrogate_weights {
   const float* d2_b;    /* [H][d] */
 } vp_surrogate_weights;
 
+/*
+ * Positional information and qk-norm of the QKV step (Algorithm 1 step (2): Q, K, V <-
+ * QKV_h(X~) with positional information P).  The paper names P but does not define it; this
+ * is the library's reading, applied in the QKV projection's epilogue before the router sees
+ * Q and K:
+ *   qk-norm: q_h <- LayerNorm_d(q_h) (.) q_norm_g + q_norm_b over each head's d channels
+ *     (biased variance, norm_eps), the [d] parameters shared by all heads; likewise k.
+ *   2-D rotary position embedding (RoFormer's rotation applied per image axis): a token's
+ *     position inside its view is (0, 0) for the patch_start special tokens and
+ *     (r + 1, c + 1) for patch r * grid_w + c.  Channels [0, d/2) rotate with the row and
+ *     [d/2, d) with the column: within a half, channels i and i + d/4 (i < d/4) turn by the
+ *     angle pos * rope_base^(-4 i / d), (a, b) -> (a cos - b sin, b cos + a sin).
+ * Tokens are numbered view after view, tokens_per_view per view.  Positions up to
+ * VP_ROPE_MAX_POS (grid rows + 1 and grid_w + 1).
+ */
+#define VP_ROPE_MAX_POS 1023
+typedef struct vp_qk_options {
+  const float* q_norm_g; const float* q_norm_b;  /* [d], or NULL: no q-norm (both or neither) */
+  const float* k_norm_g; const float* k_norm_b;  /* [d], or NULL: no k-norm */
+  float norm_eps;
+  int32_t rope;             /* 1: 2-D rotary position embedding of q and k, 0: none */
+  int32_t tokens_per_view;  /* P (N must be a multiple of it) */
+  int32_t patch_start;      /* special tokens at the start of a view (camera + registers) */
+  int32_t grid_w;           /* patches per grid row */
+  float rope_base;          /* frequency base */
+} vp_qk_options;
+
 /* One global block of Algorithm 1; matrices in the nn.Linear layout [out][in]. */
 typedef struct vp_layer_weights {
   const float* ln1_g; const float* ln1_b;       /* [D] */
@@ -121,6 +148,8 @@ typedef struct vp_layer_weights {
   const float* ls2;                             /* [D] LayerScale 2 */
   vp_router_weights router;
   vp_surrogate_weights surrogate;
+  const vp_qk_options* qk;                      /* HOST pointer: positional encoding and
+                                                   qk-norm of the QKV step, or NULL (none) */
 } vp_layer_weights;
 
 /* Workspace kinds for vp_workspace_size. */
@@ -218,11 +247,13 @@ vp_status vp_layer_norm(int32_t M, int32_t D, const vp_bf16* x, const float* gam
  *   qkv_out [N][3D] / y_out [N][D] bf16 or NULL: copies of the intermediates (debug).
  *   s_out [H] float / modes_out [H] int32 or NULL; s_attn_out [H] float or NULL: MaxAttn
  *   saliency of the full heads (see vp_head_attention).
+ *   qk: HOST pointer, positional encoding and qk-norm of the QKV step (vp_qk_options), or
+ *   NULL (none).
  */
 vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const vp_bf16* w_qkv,
                                   const float* b_qkv, const vp_bf16* w_o, const float* b_o,
                                   const vp_router_weights* rw, const vp_surrogate_weights* sw,
-                                  const int32_t* force_modes, vp_bf16* out, vp_bf16* qkv_out,
+                                  const vp_qk_options* qk, const int32_t* force_modes, vp_bf16* out, vp_bf16* qkv_out,
                                   vp_bf16* y_out, float* s_out, float* s_attn_out,
                                   int32_t* modes_out, void* ws, size_t ws_bytes, void* stream);
 

@@ -8,8 +8,8 @@ path; only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 with the CUDA path: the only common module is ``synth`` (seeded random inputs).
 
 Precision: every step runs in float64.  Where the library stores a tensor in
-bf16 (QKV, the head outputs Y, the layer output, and inside the block the
-normalised tokens, the residual stream and the FFN hidden layer) the oracle
+bf16 (QKV, the head outputs Y, the layer output, and inside the block the LN2
+output, the residual stream and the FFN hidden layer) the oracle
 rounds its float64 values to the nearest bf16 at the same point, through the
 ``materialize`` argument; pins pass ``materialize=None`` to compare against
 textbook formulations without those storage roundings.  Mode decisions compare
@@ -30,6 +30,7 @@ from .modes import (full_attention, surrogate_attention, mean_pooling, surrogate
                     max_attention_saliency, elu_feature_map, linear_attention)
 from .layer import (qkv_projection, head_router, moh_attention, global_block,
                     global_stack, load_layer, VARIANTS)
+from .position import token_positions, rope_2d, qk_transform
 
 __all__ = [
     "round_bf16", "bf16_bits_to_f64", "sigmoid", "gelu", "softmax", "layer_norm",
@@ -38,5 +39,6 @@ __all__ = [
     "full_attention", "surrogate_attention", "mean_pooling", "surrogate_mlp",
     "max_attention_saliency", "elu_feature_map", "linear_attention", "VARIANTS",
     "qkv_projection", "head_router", "moh_attention", "global_block", "global_stack",
+    "token_positions", "rope_2d", "qk_transform",
     "load_layer",
 ]

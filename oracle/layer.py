@@ -12,6 +12,7 @@ import numpy as np
 
 from .modes import full_attention, linear_attention, mean_pooling, surrogate_attention
 from .numerics import bf16_bits_to_f64, gelu, layer_norm, round_bf16
+from .position import qk_transform, token_positions
 from .router import MODE_FULL, MODE_SURROGATE, attention_pool, routing_vector, saliency, select_mode
 
 TAU_LOW = np.float32(0.01)     # §4.2 / App. B
@@ -32,16 +33,26 @@ def load_layer(w: dict) -> dict:
     return out
 
 
-def qkv_projection(Xt, lw, materialize=round_bf16):
+def qkv_projection(Xt, lw, materialize=round_bf16, qk=None):
     """Algorithm 1 step (2): (Q_h, K_h, V_h) <- QKV_h(X~).  A single linear map
     with bias whose 3D outputs are ordered (Q|K|V, head, channel); the returned
-    array is [N, 3, H, d].  Positional information P enters no synthetic
-    workload here (the paper does not define it)."""
+    array is [N, 3, H, d].  Positional information P (which the paper does not define)
+    is off unless ``qk`` gives the reading of oracle.position: a dict with "q_norm" /
+    "k_norm" ((gamma, beta) [d] or None), "eps", and "rope" (None or a dict with
+    tokens_per_view, patch_start, grid_w, base); stored in bf16 after it."""
     materialize = materialize or _identity
     N = Xt.shape[0]
     H = lw["r_W"].shape[0]
-    qkv = materialize(np.asarray(Xt, np.float64) @ lw["w_qkv"].T + lw["b_qkv"])
-    return qkv.reshape(N, 3, H, -1)
+    qkv = (np.asarray(Xt, np.float64) @ lw["w_qkv"].T + lw["b_qkv"]).reshape(N, 3, H, -1)
+    if qk is not None:
+        rope = qk.get("rope")
+        pos = None if rope is None else token_positions(N, rope["tokens_per_view"],
+                                                        rope["patch_start"], rope["grid_w"])
+        base = None if rope is None else rope["base"]
+        for h in range(H):
+            qkv[:, 0, h] = qk_transform(qkv[:, 0, h], qk.get("q_norm"), qk.get("eps", 1e-6), pos, base)
+            qkv[:, 1, h] = qk_transform(qkv[:, 1, h], qk.get("k_norm"), qk.get("eps", 1e-6), pos, base)
+    return materialize(qkv)
 
 
 # Ablation variants of §5 (component ablation and compute-mode ablation).  Two-branch
@@ -60,7 +71,7 @@ def head_router(Q_h, K_h, lw, h, beta=None, mean_qpool=False):
 
 
 def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
-                  tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=()):
+                  tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=(), qk=None):
     """Routed multi-head attention of one layer (Algorithm 1 steps 2-3 up to W_O).
 
     X [N, D] float64 (the block passes LN1(X)); lw from load_layer.
@@ -74,7 +85,7 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
     mat = materialize or _identity
     X = np.asarray(X, np.float64)
     N = X.shape[0]
-    qkv = qkv_projection(X, lw, materialize)
+    qkv = qkv_projection(X, lw, materialize, qk=qk)
     H, d = qkv.shape[2], qkv.shape[3]
     idx = np.arange(N) if rows is None else np.asarray(rows)
     res = {"qkv": qkv, "q_pool": np.zeros((H, d)), "s": np.zeros(H), "ctx": np.zeros((H, d)),
@@ -113,7 +124,7 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
 
 
 def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
-                 tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=()):
+                 tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=(), qk=None):
     """Algorithm 1 (VGGT-Prime global aggregator block), all rows.
 
     (1) X~ = LN1(X); (2) routed attention -> Y; (3) A = LS1(Y W_O),
@@ -127,7 +138,7 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
     X = np.asarray(X, np.float64)
     Xt = layer_norm(X, lw["ln1_g"], lw["ln1_b"], eps)
     att = moh_attention(Xt, lw, force_modes=force_modes, materialize=materialize,
-                        tau_low=tau_low, tau_high=tau_high, variant=variant)
+                        tau_low=tau_low, tau_high=tau_high, variant=variant, qk=qk)
     A = (att["Y"] @ lw["w_o"].T + lw["b_o"]) * lw["ls1"]
     X_attn = mat(X + A)
     Zt = mat(layer_norm(X_attn, lw["ln2_g"], lw["ln2_b"], eps))
@@ -138,13 +149,15 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
                     "s": att["s"], "X_attn": X_attn, "qkv": att["qkv"]}
 
 
-def global_stack(X, layers, force_modes=None, materialize=round_bf16, eps=LN_EPS, variant=()):
-    """Algorithm 1 applied layer after layer.  force_modes: [n_layers, H] or None.
+def global_stack(X, layers, force_modes=None, materialize=round_bf16, eps=LN_EPS, variant=(),
+                 qk=None):
+    """Algorithm 1 applied layer after layer.  force_modes: [n_layers, H] or None;
+    qk: per-layer list of qkv_projection's qk options, or None.
     Returns (X_out, list of per-layer info)."""
     infos = []
     for l, lw in enumerate(layers):
         fm = None if force_modes is None else force_modes[l]
         X, info = global_block(X, lw, force_modes=fm, materialize=materialize, eps=eps,
-                               variant=variant)
+                               variant=variant, qk=None if qk is None else qk[l])
         infos.append(info)
     return X, infos

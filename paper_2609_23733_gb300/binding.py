@@ -48,10 +48,17 @@ class VpSurrogateWeights(Structure):
     _fields_ = [(n, c_void_p) for n in ("g1_w", "g1_b", "g2_w", "g2_b", "d1_w", "d1_b", "d2_w", "d2_b")]
 
 
+class VpQkOptions(Structure):
+    _fields_ = [(n, c_void_p) for n in ("q_norm_g", "q_norm_b", "k_norm_g", "k_norm_b")] + \
+               [("norm_eps", c_float), ("rope", c_int32), ("tokens_per_view", c_int32),
+                ("patch_start", c_int32), ("grid_w", c_int32), ("rope_base", c_float)]
+
+
 class VpLayerWeights(Structure):
     _fields_ = [(n, c_void_p) for n in ("ln1_g", "ln1_b", "w_qkv", "b_qkv", "w_o", "b_o", "ls1",
                                         "ln2_g", "ln2_b", "w_fc1", "b_fc1", "w_fc2", "b_fc2", "ls2")] + \
-               [("router", VpRouterWeights), ("surrogate", VpSurrogateWeights)]
+               [("router", VpRouterWeights), ("surrogate", VpSurrogateWeights),
+                ("qk", POINTER(VpQkOptions))]
 
 
 _lib = None
@@ -78,7 +85,8 @@ _SIGS = [
                                 c_void_p]),
     ("vp_moh_global_attention", c_int32, [POINTER(VpDims), c_void_p, c_void_p, c_void_p, c_void_p,
                                           c_void_p, POINTER(VpRouterWeights),
-                                          POINTER(VpSurrogateWeights), c_void_p, c_void_p, c_void_p,
+                                          POINTER(VpSurrogateWeights), POINTER(VpQkOptions), c_void_p,
+                                          c_void_p, c_void_p,
                                           c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
                                           c_void_p]),
     ("vp_profile_begin", c_int32, [c_int32]),
@@ -141,12 +149,30 @@ def surrogate_weights(w: dict) -> VpSurrogateWeights:
                                                     "s_d1_w", "s_d1_b", "s_d2_w", "s_d2_b")])
 
 
-def layer_weights(w: dict) -> VpLayerWeights:
+def qk_options(w: dict = None, norm_eps: float = 1e-6, rope: bool = False, tokens_per_view: int = 1,
+               patch_start: int = 0, grid_w: int = 1, rope_base: float = 100.0) -> VpQkOptions:
+    """vp_qk_options from device tensors w["q_norm_g"], ... (each pair optional) and the
+    RoPE token layout."""
+    w = w or {}
+    o = VpQkOptions(*[_p(w.get(k)) for k in ("q_norm_g", "q_norm_b", "k_norm_g", "k_norm_b")])
+    o.norm_eps = norm_eps
+    o.rope = 1 if rope else 0
+    o.tokens_per_view = tokens_per_view
+    o.patch_start = patch_start
+    o.grid_w = grid_w
+    o.rope_base = rope_base
+    return o
+
+
+def layer_weights(w: dict, qk: VpQkOptions = None) -> VpLayerWeights:
     lw = VpLayerWeights(*[_p(w[k]) for k in ("ln1_g", "ln1_b", "w_qkv", "b_qkv", "w_o", "b_o", "ls1",
                                              "ln2_g", "ln2_b", "w_fc1", "b_fc1", "w_fc2", "b_fc2",
                                              "ls2")])
     lw.router = router_weights(w)
     lw.surrogate = surrogate_weights(w)
+    if qk is not None:
+        lw.qk = ctypes.pointer(qk)
+        lw._qk_keep = qk  # the struct must outlive the call
     return lw
 
 
@@ -239,9 +265,11 @@ def vp_layer_norm(x, gamma, beta, eps=1e-6, out=None, stream=None):
 
 
 def vp_moh_global_attention(dm, x, w_qkv, b_qkv, w_o, b_o, rw, sw, force_modes, out, qkv_out, y_out,
-                            s_out, modes_out, ws, stream=None, s_attn_out=None):
+                            s_out, modes_out, ws, stream=None, s_attn_out=None, qk=None):
     _check(lib().vp_moh_global_attention(ctypes.byref(dm), _p(x), _p(w_qkv), _p(b_qkv), _p(w_o), _p(b_o),
-                                         ctypes.byref(rw), ctypes.byref(sw), _p(force_modes), _p(out),
+                                         ctypes.byref(rw), ctypes.byref(sw),
+                                         ctypes.byref(qk) if qk is not None else None,
+                                         _p(force_modes), _p(out),
                                          _p(qkv_out), _p(y_out), _p(s_out), _p(s_attn_out), _p(modes_out),
                                          _p(ws), ws.numel(), _stream(stream)), "vp_moh_global_attention")
 

@@ -149,9 +149,13 @@ vp_status check_device() {
   return VP_OK;
 }
 
+// RoPE cos / sin table (vp_qk_options), [VP_ROPE_MAX_POS + 1][16] float2.
+constexpr size_t kRopeTableBytes = (size_t)(VP_ROPE_MAX_POS + 1) * 16 * sizeof(float2);
+
 size_t layer_ws_bytes(const vp_dims* dm) {
   const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
-  return heads_scratch_bytes(dm->H) + align_up(N * 3 * D * 2) + align_up(N * D * 2);
+  return heads_scratch_bytes(dm->H) + align_up(kRopeTableBytes) + align_up(N * 3 * D * 2) +
+         align_up(N * D * 2);
 }
 
 // The stack's LayerNorm scratch: LN1's row statistics (per 128-column block), the current
@@ -164,7 +168,55 @@ size_t ln_scratch_bytes(size_t N, size_t D) {
 size_t stack_ws_bytes(const vp_dims* dm) {
   const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
   // LayerNorm scratch + one region shared by {QKV, Y} and the FFN hidden layer.
-  return heads_scratch_bytes(dm->H) + ln_scratch_bytes(N, D) + align_up(N * 4 * D * 2);
+  return heads_scratch_bytes(dm->H) + align_up(kRopeTableBytes) + ln_scratch_bytes(N, D) +
+         align_up(N * 4 * D * 2);
+}
+
+// Host-side checks of vp_qk_options; *max_pos: the largest position index a token takes.
+vp_status check_qk(const vp_qk_options* qk, const vp_dims* dm, int* max_pos) {
+  *max_pos = 0;
+  if (!qk) return VP_OK;
+  if (!qk->q_norm_g != !qk->q_norm_b || !qk->k_norm_g != !qk->k_norm_b) return VP_ERR_INVALID_ARG;
+  if ((qk->q_norm_g && (!aligned16(qk->q_norm_g) || !aligned16(qk->q_norm_b))) ||
+      (qk->k_norm_g && (!aligned16(qk->k_norm_g) || !aligned16(qk->k_norm_b))))
+    return VP_ERR_ALIGNMENT;
+  if ((qk->q_norm_g || qk->k_norm_g) && !(qk->norm_eps >= 0.f)) return VP_ERR_INVALID_ARG;
+  if (qk->rope != 0 && qk->rope != 1) return VP_ERR_INVALID_ARG;
+  if (qk->rope) {
+    if (qk->tokens_per_view < 1 || qk->patch_start < 0 || qk->grid_w < 1 ||
+        qk->patch_start > qk->tokens_per_view || !(qk->rope_base > 0.f))
+      return VP_ERR_INVALID_ARG;
+    if (dm->N % qk->tokens_per_view != 0) return VP_ERR_UNSUPPORTED_SHAPE;
+    const int patches = qk->tokens_per_view - qk->patch_start;
+    const int rows = (patches + qk->grid_w - 1) / qk->grid_w;
+    *max_pos = rows > qk->grid_w ? rows : qk->grid_w;
+    if (*max_pos > VP_ROPE_MAX_POS) return VP_ERR_UNSUPPORTED_SHAPE;
+  }
+  return VP_OK;
+}
+
+// The QKV projection's qk-norm / RoPE settings and the device RoPE table.
+struct QkArgs {
+  const vp_qk_options* o;
+  const float2* table;
+};
+
+void set_qk(LinearArgs& la, const QkArgs* qk, int D) {
+  if (!qk || !qk->o) return;
+  const vp_qk_options& o = *qk->o;
+  if (!o.q_norm_g && !o.k_norm_g && !o.rope) return;
+  la.qk_cols = 2 * D;
+  la.qn_g = o.q_norm_g;
+  la.qn_b = o.q_norm_b;
+  la.kn_g = o.k_norm_g;
+  la.kn_b = o.k_norm_b;
+  la.qk_eps = o.norm_eps;
+  if (o.rope) {
+    la.rope_cs = qk->table;
+    la.tok_per_view = o.tokens_per_view;
+    la.patch_start = o.patch_start;
+    la.grid_w = o.grid_w;
+  }
 }
 
 // Row widths the LayerNorm kernel is instantiated for.
@@ -269,7 +321,7 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
                     const vp_surrogate_weights* sw, const int32_t* force_modes,
                     __nv_bfloat16* out, __nv_bfloat16* qkv, __nv_bfloat16* y, float* s_out,
                     float* s_attn_out, int32_t* modes_out, const RouterScratch& sc,
-                    cudaStream_t st, const LnFold* fold = nullptr) {
+                    cudaStream_t st, const LnFold* fold = nullptr, const QkArgs* qk = nullptr) {
   const int N = dm->N, D = dm->H * kHeadDim;
   const int sms = device_sm_count();
   LinearArgs la{};
@@ -287,6 +339,7 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
     la.ln_c = fold->c;
     la.ln_eps = fold->eps;
   }
+  set_qk(la, qk, D);
   VP_TRY(from_cuda(launch_linear(la, sms, st)));
   RouterArgs ra = make_router_args(dm, reinterpret_cast<const vp_bf16*>(qkv), rw, force_modes);
   ra.s_out = s_out;
@@ -491,9 +544,10 @@ vp_status vp_layer_norm(int32_t M, int32_t D, const vp_bf16* x, const float* gam
 vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const vp_bf16* w_qkv,
                                   const float* b_qkv, const vp_bf16* w_o, const float* b_o,
                                   const vp_router_weights* rw, const vp_surrogate_weights* sw,
-                                  const int32_t* force_modes, vp_bf16* out, vp_bf16* qkv_out,
-                                  vp_bf16* y_out, float* s_out, float* s_attn_out,
-                                  int32_t* modes_out, void* ws, size_t ws_bytes, void* stream) {
+                                  const vp_qk_options* qk, const int32_t* force_modes,
+                                  vp_bf16* out, vp_bf16* qkv_out, vp_bf16* y_out, float* s_out,
+                                  float* s_attn_out, int32_t* modes_out, void* ws, size_t ws_bytes,
+                                  void* stream) {
   VP_TRY(check_dims(dims));
   if (!x || !w_qkv || !w_o || !out) return VP_ERR_INVALID_ARG;
   if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(w_o) || !aligned16(out) ||
@@ -502,12 +556,18 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
     return VP_ERR_ALIGNMENT;
   VP_TRY(check_router_weights(rw));
   VP_TRY(check_surrogate_weights(sw));
+  int max_pos = 0;
+  VP_TRY(check_qk(qk, dims, &max_pos));
   if (!ws || ws_bytes < layer_ws_bytes(dims)) return VP_ERR_WORKSPACE;
   VP_TRY(check_device());
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t N = dims->N, D = (size_t)dims->H * kHeadDim;
   RouterScratch sc = carve_router_scratch(ws, dims->H);
   char* p = static_cast<char*>(ws) + heads_scratch_bytes(dims->H);
+  float2* rope = reinterpret_cast<float2*>(p);
+  p += align_up(kRopeTableBytes);
+  if (qk && qk->rope) VP_TRY(from_cuda(launch_rope_table(max_pos, qk->rope_base, rope, st)));
+  const QkArgs qa{qk, rope};
   __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
   p += align_up(N * 3 * D * 2);
   __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p);
@@ -515,7 +575,7 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
   if (y_out) y = reinterpret_cast<__nv_bfloat16*>(y_out);
   return run_layer(dims, reinterpret_cast<const __nv_bfloat16*>(x), w_qkv, b_qkv, w_o, b_o,
                    nullptr, nullptr, rw, sw, force_modes, reinterpret_cast<__nv_bfloat16*>(out),
-                   qkv, y, s_out, s_attn_out, modes_out, sc, st);
+                   qkv, y, s_out, s_attn_out, modes_out, sc, st, nullptr, &qa);
 }
 
 vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
@@ -540,6 +600,8 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
       return VP_ERR_ALIGNMENT;
     VP_TRY(check_router_weights(&w.router));
     VP_TRY(check_surrogate_weights(&w.surrogate));
+    int max_pos = 0;
+    VP_TRY(check_qk(w.qk, dims, &max_pos));
   }
   if (!ws || ws_bytes < stack_ws_bytes(dims)) return VP_ERR_WORKSPACE;
   VP_TRY(check_device());
@@ -547,6 +609,9 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
   const size_t N = dims->N;
   RouterScratch sc = carve_router_scratch(ws, dims->H);
   char* p = static_cast<char*>(ws) + heads_scratch_bytes(dims->H);
+  float2* rope = reinterpret_cast<float2*>(p);
+  p += align_up(kRopeTableBytes);
+  const vp_qk_options* rope_built = nullptr;  // the options the table was last built for
   // LayerNorm scratch (see ln_scratch_bytes).  LN1 is folded into the QKV projection, which
   // then reads the raw residual stream; its row statistics come from the kernel that last
   // wrote the stream (the previous block's FFN-down, or a statistics pass for the first
@@ -573,6 +638,16 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     VP_TRY(from_cuda(launch_ln_fold_weights(3 * D, D,
                                             reinterpret_cast<const __nv_bfloat16*>(w.w_qkv),
                                             w.ln1_g, w.ln1_b, w.b_qkv, wq, cq, bq, st)));
+    if (w.qk && w.qk->rope &&
+        !(rope_built && rope_built->rope_base == w.qk->rope_base &&
+          rope_built->tokens_per_view == w.qk->tokens_per_view &&
+          rope_built->patch_start == w.qk->patch_start && rope_built->grid_w == w.qk->grid_w)) {
+      int max_pos = 0;
+      VP_TRY(check_qk(w.qk, dims, &max_pos));
+      VP_TRY(from_cuda(launch_rope_table(max_pos, w.qk->rope_base, rope, st)));
+      rope_built = w.qk;
+    }
+    const QkArgs qa{w.qk, rope};
     // (1)-(3) X <- X + LS1 (Y W_O + b_O) in place, Y the routed attention of LN1(X)
     const LnFold fold{part, cq, ln_eps};
     VP_TRY(run_layer(dims, x, reinterpret_cast<const vp_bf16*>(wq), bq, w.w_o, w.b_o, w.ls1, x,
@@ -580,7 +655,8 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
                      force_modes ? force_modes + (size_t)l * dims->H : nullptr, x, qkv, y,
                      s_out ? s_out + (size_t)l * dims->H : nullptr,
                      s_attn_out ? s_attn_out + (size_t)l * dims->H : nullptr,
-                     modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st, &fold));
+                     modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st, &fold,
+                     &qa));
     // (4) Z~ = LN2(X_attn); X <- X_attn + LS2 FFN(Z~)
     VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, zt, st)));
     LinearArgs f1{};

@@ -49,6 +49,14 @@ struct GemmParams {
   const float* ln_c;
   float ln_eps;
   float2* part_out;
+  int qk_cols;  // > 0: the first qk_cols columns are Q | K of a QKV projection (see LinearArgs)
+  const float* qn_g;
+  const float* qn_b;
+  const float* kn_g;
+  const float* kn_b;
+  float qk_eps;
+  const float2* rope_cs;
+  int tok_per_view, patch_start, grid_w;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -221,6 +229,146 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       float cmean[4], cm2[4];  // output statistics per 32-column chunk (part_out)
       const uint32_t tcol = t_lane + ab * kBN + half * 128;
+      // Bias, or the folded LayerNorm rstd (acc - mu c) + bias', on one 32-column chunk.
+      auto bias_fold = [&](float* x, int col0) {
+        if (prm.ln_part) {  // rstd (acc - mu c) + bias'
+          const float2 nmu = make_float2(-ln_mu, -ln_mu), rs = make_float2(ln_rstd, ln_rstd);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const bool in = col0 + 4 * q + 3 < N;
+            const float4 c4 = in ? __ldg(reinterpret_cast<const float4*>(prm.ln_c + col0) + q)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 b4 = in ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float2 a0 = ffma2(rs, ffma2(nmu, make_float2(c4.x, c4.y),
+                                              make_float2(x[4 * q], x[4 * q + 1])),
+                                    make_float2(b4.x, b4.y));
+            const float2 a1 = ffma2(rs, ffma2(nmu, make_float2(c4.z, c4.w),
+                                              make_float2(x[4 * q + 2], x[4 * q + 3])),
+                                    make_float2(b4.z, b4.w));
+            x[4 * q] = a0.x;
+            x[4 * q + 1] = a0.y;
+            x[4 * q + 2] = a1.x;
+            x[4 * q + 3] = a1.y;
+          }
+        } else if (prm.bias) {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 b4 = col0 + 4 * q + 3 < N
+                                  ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float2 a0 = fadd2(make_float2(x[4 * q], x[4 * q + 1]), make_float2(b4.x, b4.y));
+            const float2 a1 = fadd2(make_float2(x[4 * q + 2], x[4 * q + 3]), make_float2(b4.z, b4.w));
+            x[4 * q] = a0.x;
+            x[4 * q + 1] = a0.y;
+            x[4 * q + 2] = a1.x;
+            x[4 * q + 3] = a1.y;
+          }
+        }
+      };
+      // Stage a 32 x 32 block (row = lane, 64 bytes) and write it with a TMA tensor store.
+      auto store_chunk = [&](const float* x, int col0) {
+        // Stage the 32 x 32 block (row = lane, 64 bytes) in the 64-byte swizzle the
+        // output tensor map uses: 16-byte chunk q of row r sits at chunk q ^ ((r >> 1) & 3).
+        unsigned char* buf = stg + (nst & 1) * 2048;
+        // The elected lane (lane 0, the lowest) owns this warp's bulk stores and their groups.
+        if (nst >= 2 && elect_one()) tma_store_wait_read<1>();  // this buffer's last store read it
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint4 u;
+          u.x = pack_bf16x2(x[8 * q + 0], x[8 * q + 1]);
+          u.y = pack_bf16x2(x[8 * q + 2], x[8 * q + 3]);
+          u.z = pack_bf16x2(x[8 * q + 4], x[8 * q + 5]);
+          u.w = pack_bf16x2(x[8 * q + 6], x[8 * q + 7]);
+          *reinterpret_cast<uint4*>(buf + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = u;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (elect_one()) {
+          tma_store_2d(&tmap_out, buf, col0, row0);
+          tma_store_commit();
+        }
+        ++nst;
+      };
+      const int pcol0 = nt * kBN + half * 128;  // this thread's 128 columns: two heads
+      if (prm.qk_cols > 0 && pcol0 < prm.qk_cols) {
+        // Q or K columns of a QKV projection with qk-norm and / or 2-D RoPE: whole heads
+        // (64 columns, two chunks) at a time.
+        const bool is_q = pcol0 < (prm.qk_cols >> 1);
+        const float* ng = is_q ? prm.qn_g : prm.kn_g;
+        const float* nbv = is_q ? prm.qn_b : prm.kn_b;
+        int py = 0, px = 0;  // the row's position inside its view
+        if (prm.rope_cs) {
+          const int t = row % prm.tok_per_view - prm.patch_start;
+          if (t >= 0) {
+            py = t / prm.grid_w + 1;
+            px = t - (py - 1) * prm.grid_w + 1;
+          }
+        }
+#pragma unroll 1
+        for (int hh = 0; hh < 2; ++hh) {
+          float x[64];
+          tmem_ld32(tcol + 64 * hh, x);
+          tmem_ld32(tcol + 64 * hh + 32, x + 32);
+          tmem_wait_ld();
+          if (hh == 1) {
+            tc_fence_before();
+            mbar_arrive(&sm.acc_empty[ab]);
+          }
+          const int col0 = pcol0 + 64 * hh;
+          bias_fold(x, col0);
+          bias_fold(x + 32, col0 + 32);
+          if (ng) {  // LayerNorm over the head's 64 channels
+            float2 s2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) s2 = fadd2(s2, make_float2(x[2 * k], x[2 * k + 1]));
+            const float mean = (s2.x + s2.y) * (1.f / 64.f);
+            float2 q2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const float2 dd = fadd2(make_float2(x[2 * k], x[2 * k + 1]), make_float2(-mean, -mean));
+              q2 = ffma2(dd, dd, q2);
+            }
+            const float rstd = rsqrtf((q2.x + q2.y) * (1.f / 64.f) + prm.qk_eps);
+            const float2 nm = make_float2(-mean * rstd, -mean * rstd), rs = make_float2(rstd, rstd);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+              const float4 g4 = __ldg(reinterpret_cast<const float4*>(ng) + q);
+              const float4 b4 = __ldg(reinterpret_cast<const float4*>(nbv) + q);
+              const float2 a0 = ffma2(ffma2(make_float2(x[4 * q], x[4 * q + 1]), rs, nm),
+                                      make_float2(g4.x, g4.y), make_float2(b4.x, b4.y));
+              const float2 a1 = ffma2(ffma2(make_float2(x[4 * q + 2], x[4 * q + 3]), rs, nm),
+                                      make_float2(g4.z, g4.w), make_float2(b4.z, b4.w));
+              x[4 * q] = a0.x;
+              x[4 * q + 1] = a0.y;
+              x[4 * q + 2] = a1.x;
+              x[4 * q + 3] = a1.y;
+            }
+          }
+          if (prm.rope_cs) {  // channels [0, 32) turn with the row, [32, 64) with the column
+#pragma unroll
+            for (int ax = 0; ax < 2; ++ax) {
+              const float4* cs = reinterpret_cast<const float4*>(prm.rope_cs + (size_t)(ax ? px : py) * 16);
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {  // frequencies 2q, 2q + 1: (cos, sin) pairs
+                const float4 t4 = __ldg(cs + q);
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                  const int i = 32 * ax + 2 * q + e;
+                  const float c = e ? t4.z : t4.x, sn = e ? t4.w : t4.y;
+                  const float a = x[i], b = x[i + 16];
+                  x[i] = fmaf(a, c, -b * sn);
+                  x[i + 16] = fmaf(b, c, a * sn);
+                }
+              }
+            }
+          }
+          if (col0 < N) store_chunk(x, col0);
+          if (col0 + 32 < N) store_chunk(x + 32, col0 + 32);
+        }
+        continue;
+      }
       float v[2][32];
       tmem_ld32(tcol, v[0]);
       tmem_wait_ld();
@@ -231,40 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int col0 = nt * kBN + half * 128 + cc * 32;
         if (col0 < N) {
           // Bias, GELU, LayerScale and residual on column pairs (packed f32x2 arithmetic).
-          if (prm.ln_part) {  // rstd (acc - mu c) + bias'
-            const float2 nmu = make_float2(-ln_mu, -ln_mu), rs = make_float2(ln_rstd, ln_rstd);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const bool in = col0 + 4 * q + 3 < N;
-              const float4 c4 = in ? __ldg(reinterpret_cast<const float4*>(prm.ln_c + col0) + q)
-                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-              const float4 b4 = in ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
-                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-              const float2 a0 = ffma2(rs, ffma2(nmu, make_float2(c4.x, c4.y),
-                                                make_float2(x[4 * q], x[4 * q + 1])),
-                                      make_float2(b4.x, b4.y));
-              const float2 a1 = ffma2(rs, ffma2(nmu, make_float2(c4.z, c4.w),
-                                                make_float2(x[4 * q + 2], x[4 * q + 3])),
-                                      make_float2(b4.z, b4.w));
-              x[4 * q] = a0.x;
-              x[4 * q + 1] = a0.y;
-              x[4 * q + 2] = a1.x;
-              x[4 * q + 3] = a1.y;
-            }
-          } else if (prm.bias) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const float4 b4 = col0 + 4 * q + 3 < N
-                                    ? __ldg(reinterpret_cast<const float4*>(prm.bias + col0) + q)
-                                    : make_float4(0.f, 0.f, 0.f, 0.f);
-              const float2 a0 = fadd2(make_float2(x[4 * q], x[4 * q + 1]), make_float2(b4.x, b4.y));
-              const float2 a1 = fadd2(make_float2(x[4 * q + 2], x[4 * q + 3]), make_float2(b4.z, b4.w));
-              x[4 * q] = a0.x;
-              x[4 * q + 1] = a0.y;
-              x[4 * q + 2] = a1.x;
-              x[4 * q + 3] = a1.y;
-            }
-          }
+          bias_fold(x, col0);
           if (prm.act == VP_ACT_GELU) {
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
@@ -318,28 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             cmean[cc] = cm;
             cm2[cc] = q2.x + q2.y;
           }
-          // Stage the 32 x 32 block (row = lane, 64 bytes) in the 64-byte swizzle the
-          // output tensor map uses: 16-byte chunk q of row r sits at chunk q ^ ((r >> 1) & 3).
-          unsigned char* buf = stg + (nst & 1) * 2048;
-          // The elected lane (lane 0, the lowest) owns this warp's bulk stores and their groups.
-          if (nst >= 2 && elect_one()) tma_store_wait_read<1>();  // this buffer's last store read it
-          __syncwarp();
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            uint4 u;
-            u.x = pack_bf16x2(x[8 * q + 0], x[8 * q + 1]);
-            u.y = pack_bf16x2(x[8 * q + 2], x[8 * q + 3]);
-            u.z = pack_bf16x2(x[8 * q + 4], x[8 * q + 5]);
-            u.w = pack_bf16x2(x[8 * q + 6], x[8 * q + 7]);
-            *reinterpret_cast<uint4*>(buf + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = u;
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (elect_one()) {
-            tma_store_2d(&tmap_out, buf, col0, row0);
-            tma_store_commit();
-          }
-          ++nst;
+          store_chunk(x, col0);
         }
         tmem_wait_ld();
         if (cc == 3) {
@@ -368,7 +462,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// RoPE angles in double precision: table[p][i] = (cos, sin)(p base^(-i / 16)).
+__global__ void rope_table_kernel(int max_pos, double base, float2* table) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= (max_pos + 1) * 16) return;
+  const int p = k >> 4, i = k & 15;
+  double sn, cs;
+  sincos((double)p * pow(base, -(double)i / 16.0), &sn, &cs);
+  table[k] = make_float2((float)cs, (float)sn);
+}
+
 }  // namespace
+
+cudaError_t launch_rope_table(int max_pos, float base, float2* table, cudaStream_t st) {
+  const int n = (max_pos + 1) * 16;
+  rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(max_pos, (double)base, table);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   CUtensorMap ta, tb, to;
@@ -385,8 +495,15 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   if ((a.ln_part && (a.K % 256 != 0 || !a.ln_c || !a.bias)) ||
       (a.part_out && a.N % 128 != 0))
     return cudaErrorInvalidValue;
+  const bool qk = a.qk_cols > 0;
+  if (qk && (a.qk_cols % 256 != 0 || a.qk_cols > a.N || a.act != VP_ACT_NONE || a.scale ||
+             a.residual || a.part_out || (!a.qn_g != !a.qn_b) || (!a.kn_g != !a.kn_b) ||
+             (a.rope_cs && (a.tok_per_view < 1 || a.grid_w < 1 || a.patch_start < 0))))
+    return cudaErrorInvalidValue;
   GemmParams prm{a.M,     a.N,   a.K,   a.bias,      a.act,  a.scale,   a.residual,
-                 a.out,   a.err, a.ln_part, a.ln_c, a.ln_eps, a.part_out};
+                 a.out,   a.err, a.ln_part, a.ln_c, a.ln_eps, a.part_out,
+                 qk ? a.qk_cols : 0, a.qn_g, a.qn_b, a.kn_g, a.kn_b, a.qk_eps, a.rope_cs,
+                 a.tok_per_view, a.patch_start, a.grid_w};
   prof_before(VP_KERNEL_GEMM, st);
   gemm_kernel<<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
   prof_after(st);

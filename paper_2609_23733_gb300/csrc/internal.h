@@ -135,6 +135,18 @@ struct LinearArgs {
   const float* ln_c;      // [N] column sums of W'
   float ln_eps;
   float2* part_out;       // [M][N / 128] (mean, M2) blocks of the output rows, or NULL (N % 128 == 0)
+  // QKV projection with qk-norm and / or 2-D RoPE (vp_qk_options) on its first qk_cols = 2D
+  // columns (Q | K; a multiple of 256, so a tile half holds two whole heads of Q or of K):
+  // LayerNorm over each head's 64 channels with qn_* / kn_* ([64], NULL: none), then the
+  // rotation by rope_cs [pos][16] (cos, sin) at the token's (row, column) position.
+  int qk_cols;
+  const float* qn_g;
+  const float* qn_b;
+  const float* kn_g;
+  const float* kn_b;
+  float qk_eps;
+  const float2* rope_cs;  // NULL: no RoPE
+  int tok_per_view, patch_start, grid_w;
 };
 cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st);
 
@@ -144,6 +156,8 @@ cudaError_t launch_ln_partials(int M, int D, const __nv_bfloat16* x, float2* par
 // The folded LayerNorm's weights for a projection W [Nout][K] (nn.Linear layout):
 // Wp = W diag(g) (bf16), c[o] = sum_k Wp[o][k] (of the bf16 Wp), bp[o] = b[o] + sum_k W[o][k] beta[k]
 // (b NULL: 0).  K % 256 == 0, K <= 4096.
+// cos / sin of p * base^(-i / 16), p = 0 .. max_pos, i = 0 .. 15: table [max_pos + 1][16].
+cudaError_t launch_rope_table(int max_pos, float base, float2* table, cudaStream_t st);
 cudaError_t launch_ln_fold_weights(int Nout, int K, const __nv_bfloat16* W, const float* g,
                                    const float* beta, const float* b, __nv_bfloat16* Wp,
                                    float* c, float* bp, cudaStream_t st);

@@ -95,6 +95,17 @@ def make_tokens(seed: int, N: int, D: int = D_MODEL) -> np.ndarray:
     return f32_to_bf16_bits(g.standard_normal((N, D), dtype=np.float32))
 
 
+def make_qk_norm_weights(g: np.random.Generator, *, d: int = HEAD_DIM, jitter: float = 0.1,
+                         bias_std: float = 0.05) -> dict:
+    """qk-norm parameters (per-channel LayerNorm scale and shift of q and k, shared by the
+    heads), float32: q_norm_g, q_norm_b, k_norm_g, k_norm_b."""
+    w = {}
+    for t in ("q", "k"):
+        w[f"{t}_norm_g"] = (1.0 + jitter * g.standard_normal(d)).astype(np.float32)
+        w[f"{t}_norm_b"] = (bias_std * g.standard_normal(d)).astype(np.float32)
+    return w
+
+
 def make_layer_weights(g: np.random.Generator, *, D: int = D_MODEL, H: int = N_HEADS,
                        d: int = HEAD_DIM, L: int = HIDDEN, block: bool = False,
                        bias_std: float = 0.0, norm_jitter: float = 0.0) -> dict:
