@@ -384,6 +384,8 @@ def run_ours(args):
         line["cheap_mode_variants"] = variant_probe(vpb, dev, N, dws[0], pk)
     if args.qk:
         line["qkv_positional"] = qk_probe(vpb, dev, N, dws[0])
+    if args.tome:
+        line["token_merging_s100"] = tome_probe(vpb, dev, N, dws, fm)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
@@ -460,6 +462,45 @@ def variant_probe(vpb, dev, N, dw, pk):
         gbs = bytes_per_token * N * H / (ms * 1e-3) / 1e9
         out[name] = {"ms_16_heads": ms, "gb_s": gbs, "hbm_frac": gbs / hbm}
     out["tokens"] = N
+    return out
+
+
+def tome_probe(vpb, dev, N, dws, fm, steps=3, warmup=2):
+    """The S = 100 stack with token merging in every block (vp_merge_options: stride 4 merges
+    ~75 % of the tokens, stride 10 ~90 %; the paper's "VGGT-Prime & Token Merging"), same
+    weights and routes as the headline run."""
+    import torch
+    P = synth.tokens_per_view(518)
+    L = len(dws)
+    x0 = vpb.bf16_from_bits(synth.make_tokens(WORKLOAD.seed, N), dev)
+    x = torch.empty_like(x0)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE, dev)
+    modes = torch.zeros(L, H, dtype=torch.int32, device=dev)
+    s = torch.zeros(L, H, device=dev)
+    out = {}
+    for stride in (4, 10):
+        layers = [vpb.layer_weights(w, None, vpb.merge_options(stride, P, 5)) for w in dws]
+        n_rows = P + (N // P - 1) * (5 + -(-(P - 5) // stride))
+
+        def step():
+            x.copy_(x0)
+            vpb.vp_global_stack(dm, x, layers, fm, modes, s, 1e-6, ws)
+        for _ in range(warmup):
+            step()
+        torch.cuda.synchronize()
+        vpb.vp_profile_begin(96 * L * steps)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            step()
+        b.record()
+        torch.cuda.synchronize()
+        _, cnt, ms = vpb.vp_profile_end()
+        t = a.elapsed_time(b) / steps
+        out[f"stride_{stride}"] = {"merged_fraction": 1 - n_rows / N, "merged_tokens": n_rows,
+                                   "ms_per_forward": t, "views_per_s": WORKLOAD.views / t * 1e3,
+                                   "kernels_ms": {k: v / steps for k, v in ms.items() if cnt[k]}}
     return out
 
 
@@ -639,6 +680,7 @@ def main():
     ap.add_argument("--variants", action="store_true", default=True)
     ap.add_argument("--no-variants", dest="variants", action="store_false")
     ap.add_argument("--no-qk", dest="qk", action="store_false")
+    ap.add_argument("--no-tome", dest="tome", action="store_false")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
                                               "surrogate", "mean", "bin"],
                     default=None,

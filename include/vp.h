@@ -136,6 +136,30 @@ typedef struct vp_qk_options {
   float rope_base;          /* frequency base */
 } vp_qk_options;
 
+/*
+ * Token merging around a block's attention (the paper's "VGGT-Prime & Token Merging": ToMe as
+ * used by FastVGGT, 75 % or 90 % of the tokens merged; the paper gives no further detail, so
+ * this is the library's reading, applied to LN1(X) of a block of vp_global_stack):
+ *   destinations: the patch_start special tokens of every view, every token of the first
+ *     view, and patch tokens p % stride == 0 of the other views; all others are sources
+ *     (stride 4 merges ~75 % of the tokens, 10 ~90 %);
+ *   metric: the head mean of the block's keys, mean_h (x~ W_k,h^T + b_k,h), as a unit vector;
+ *   matching: every source joins the destination of largest cosine similarity over all
+ *     destinations (ties: lowest merged row);
+ *   merged token: the mean of a destination and the sources that joined it; the routed
+ *     attention (QKV, router, modes, W_O) runs on the merged tokens in destination order,
+ *     positions (vp_qk_options) taken from each destination's own token;
+ *   unmerge: X_i += LS1 (.) A[merged row of i] for every token.
+ * tokens_per_view must divide N.  assign_out: [N] int32 device buffer receiving the merged row
+ * every token joined, or NULL.
+ */
+typedef struct vp_merge_options {
+  int32_t stride;
+  int32_t tokens_per_view;
+  int32_t patch_start;
+  int32_t* assign_out;
+} vp_merge_options;
+
 /* One global block of Algorithm 1; matrices in the nn.Linear layout [out][in]. */
 typedef struct vp_layer_weights {
   const float* ln1_g; const float* ln1_b;       /* [D] */
@@ -150,12 +174,15 @@ typedef struct vp_layer_weights {
   vp_surrogate_weights surrogate;
   const vp_qk_options* qk;                      /* HOST pointer: positional encoding and
                                                    qk-norm of the QKV step, or NULL (none) */
+  const vp_merge_options* merge;                /* HOST pointer: token merging around the
+                                                   block's attention, or NULL (none) */
 } vp_layer_weights;
 
 /* Workspace kinds for vp_workspace_size. */
 #define VP_WS_ROUTER 0   /* vp_router, vp_head_attention (router scratch + linear-attention state) */
 #define VP_WS_LAYER 1    /* vp_moh_global_attention */
 #define VP_WS_STACK 2    /* vp_global_stack */
+#define VP_WS_STACK_MERGE 3  /* vp_global_stack with token merging in some block */
 
 /* Epilogues of vp_linear. */
 #define VP_ACT_NONE 0
@@ -303,8 +330,10 @@ vp_status vp_router_noalloc(const vp_dims* dims, const vp_bf16* qkv, const vp_ro
                                    kernel overlapping its tail, timed as one bracket */
 #define VP_KERNEL_SURROGATE 6   /* (unused: surrogate and mean heads are timed with class 5) */
 #define VP_KERNEL_MEAN 7
-#define VP_KERNEL_LAYER_NORM 8
-#define VP_KERNEL_CLASSES 9
+#define VP_KERNEL_LAYER_NORM 8  /* LayerNorm, and the stack's LN1 statistics pass and QKV
+                                   weight fold */
+#define VP_KERNEL_MERGE 9       /* token merging (vp_merge_options) and the unmerge */
+#define VP_KERNEL_CLASSES 10
 
 /*
  * Launch profiler (for benchmarks; not part of the method).  Between vp_profile_begin and

@@ -31,6 +31,7 @@ from .modes import (full_attention, surrogate_attention, mean_pooling, surrogate
 from .layer import (qkv_projection, head_router, moh_attention, global_block,
                     global_stack, load_layer, VARIANTS)
 from .position import token_positions, rope_2d, qk_transform
+from .merge import destinations, key_metric, match, merge_tokens
 
 __all__ = [
     "round_bf16", "bf16_bits_to_f64", "sigmoid", "gelu", "softmax", "layer_norm",
@@ -39,6 +40,7 @@ __all__ = [
     "full_attention", "surrogate_attention", "mean_pooling", "surrogate_mlp",
     "max_attention_saliency", "elu_feature_map", "linear_attention", "VARIANTS",
     "qkv_projection", "head_router", "moh_attention", "global_block", "global_stack",
-    "token_positions", "rope_2d", "qk_transform",
+    "token_positions", "rope_2d", "qk_transform", "destinations", "key_metric", "match",
+    "merge_tokens",
     "load_layer",
 ]

@@ -12,6 +12,7 @@ import numpy as np
 
 from .modes import full_attention, linear_attention, mean_pooling, surrogate_attention
 from .numerics import bf16_bits_to_f64, gelu, layer_norm, round_bf16
+from .merge import destinations, key_metric, match, merge_tokens
 from .position import qk_transform, token_positions
 from .router import MODE_FULL, MODE_SURROGATE, attention_pool, routing_vector, saliency, select_mode
 
@@ -33,21 +34,26 @@ def load_layer(w: dict) -> dict:
     return out
 
 
-def qkv_projection(Xt, lw, materialize=round_bf16, qk=None):
+def qkv_projection(Xt, lw, materialize=round_bf16, qk=None, tok_index=None):
     """Algorithm 1 step (2): (Q_h, K_h, V_h) <- QKV_h(X~).  A single linear map
     with bias whose 3D outputs are ordered (Q|K|V, head, channel); the returned
     array is [N, 3, H, d].  Positional information P (which the paper does not define)
     is off unless ``qk`` gives the reading of oracle.position: a dict with "q_norm" /
     "k_norm" ((gamma, beta) [d] or None), "eps", and "rope" (None or a dict with
-    tokens_per_view, patch_start, grid_w, base); stored in bf16 after it."""
+    tokens_per_view, patch_start, grid_w, base); stored in bf16 after it.  tok_index: the
+    token each row stands for (merged tokens), positions are that token's."""
     materialize = materialize or _identity
     N = Xt.shape[0]
     H = lw["r_W"].shape[0]
     qkv = (np.asarray(Xt, np.float64) @ lw["w_qkv"].T + lw["b_qkv"]).reshape(N, 3, H, -1)
     if qk is not None:
         rope = qk.get("rope")
-        pos = None if rope is None else token_positions(N, rope["tokens_per_view"],
-                                                        rope["patch_start"], rope["grid_w"])
+        pos = None
+        if rope is not None:
+            toks = np.arange(N) if tok_index is None else np.asarray(tok_index)
+            py, px = token_positions(int(toks.max()) + 1, rope["tokens_per_view"], rope["patch_start"],
+                                     rope["grid_w"])
+            pos = (py[toks], px[toks])
         base = None if rope is None else rope["base"]
         for h in range(H):
             qkv[:, 0, h] = qk_transform(qkv[:, 0, h], qk.get("q_norm"), qk.get("eps", 1e-6), pos, base)
@@ -71,7 +77,7 @@ def head_router(Q_h, K_h, lw, h, beta=None, mean_qpool=False):
 
 
 def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
-                  tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=(), qk=None):
+                  tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=(), qk=None, tok_index=None):
     """Routed multi-head attention of one layer (Algorithm 1 steps 2-3 up to W_O).
 
     X [N, D] float64 (the block passes LN1(X)); lw from load_layer.
@@ -85,7 +91,7 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
     mat = materialize or _identity
     X = np.asarray(X, np.float64)
     N = X.shape[0]
-    qkv = qkv_projection(X, lw, materialize, qk=qk)
+    qkv = qkv_projection(X, lw, materialize, qk=qk, tok_index=tok_index)
     H, d = qkv.shape[2], qkv.shape[3]
     idx = np.arange(N) if rows is None else np.asarray(rows)
     res = {"qkv": qkv, "q_pool": np.zeros((H, d)), "s": np.zeros(H), "ctx": np.zeros((H, d)),
@@ -124,7 +130,7 @@ def moh_attention(X, lw, force_modes=None, rows=None, materialize=round_bf16,
 
 
 def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
-                 tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=(), qk=None):
+                 tau_low=TAU_LOW, tau_high=TAU_HIGH, variant=(), qk=None, merge=None, assign=None):
     """Algorithm 1 (VGGT-Prime global aggregator block), all rows.
 
     (1) X~ = LN1(X); (2) routed attention -> Y; (3) A = LS1(Y W_O),
@@ -133,31 +139,52 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
 
     Storage points (materialize, bf16): QKV, Y, Z~, the FFN hidden layer and the residual
     stream X_attn, X'.  The LN1 output X~ is not stored: the block feeds it straight into
-    the QKV projection."""
+    the QKV projection.
+
+    merge: token merging around the attention (oracle.merge; a dict with stride,
+    tokens_per_view, patch_start): X~ (stored) is merged, the routed attention and W_O (+ b_O,
+    stored) run on the merged tokens, and every token adds LS1 times its merged token's
+    output.  assign: the merged row of every token to use instead of the oracle's matching
+    (the library's choice, for parity downstream of a near-tie)."""
     mat = materialize or _identity
     X = np.asarray(X, np.float64)
     Xt = layer_norm(X, lw["ln1_g"], lw["ln1_b"], eps)
-    att = moh_attention(Xt, lw, force_modes=force_modes, materialize=materialize,
-                        tau_low=tau_low, tau_high=tau_high, variant=variant, qk=qk)
-    A = (att["Y"] @ lw["w_o"].T + lw["b_o"]) * lw["ls1"]
+    merged = None
+    if merge is not None:
+        Xt = mat(Xt)
+        row_of, dst_tok = destinations(X.shape[0], merge["tokens_per_view"], merge["patch_start"],
+                                       merge["stride"])
+        own, scores = match(key_metric(Xt, lw, mat), row_of, dst_tok)
+        asg = own if assign is None else np.asarray(assign)
+        Xm = mat(merge_tokens(Xt, asg, len(dst_tok)))
+        att = moh_attention(Xm, lw, force_modes=force_modes, materialize=materialize, tau_low=tau_low,
+                            tau_high=tau_high, variant=variant, qk=qk, tok_index=dst_tok)
+        A = att["out"][asg] * lw["ls1"]
+        merged = {"assign": own, "scores": scores, "dst_tok": dst_tok}
+    else:
+        att = moh_attention(Xt, lw, force_modes=force_modes, materialize=materialize,
+                            tau_low=tau_low, tau_high=tau_high, variant=variant, qk=qk)
+        A = (att["Y"] @ lw["w_o"].T + lw["b_o"]) * lw["ls1"]
     X_attn = mat(X + A)
     Zt = mat(layer_norm(X_attn, lw["ln2_g"], lw["ln2_b"], eps))
     Hd = mat(gelu(Zt @ lw["w_fc1"].T + lw["b_fc1"]))
     F = (Hd @ lw["w_fc2"].T + lw["b_fc2"]) * lw["ls2"]
     X_next = mat(X_attn + F)
     return X_next, {"modes": att["modes"], "natural_modes": att["natural_modes"],
-                    "s": att["s"], "X_attn": X_attn, "qkv": att["qkv"]}
+                    "s": att["s"], "X_attn": X_attn, "qkv": att["qkv"], "merge": merged}
 
 
 def global_stack(X, layers, force_modes=None, materialize=round_bf16, eps=LN_EPS, variant=(),
-                 qk=None):
+                 qk=None, merge=None, assign=None):
     """Algorithm 1 applied layer after layer.  force_modes: [n_layers, H] or None;
-    qk: per-layer list of qkv_projection's qk options, or None.
+    qk, merge, assign: per-layer lists of global_block's options, or None.
     Returns (X_out, list of per-layer info)."""
     infos = []
     for l, lw in enumerate(layers):
         fm = None if force_modes is None else force_modes[l]
         X, info = global_block(X, lw, force_modes=fm, materialize=materialize, eps=eps,
-                               variant=variant, qk=None if qk is None else qk[l])
+                               variant=variant, qk=None if qk is None else qk[l],
+                               merge=None if merge is None else merge[l],
+                               assign=None if assign is None else assign[l])
         infos.append(info)
     return X, infos

@@ -17,12 +17,12 @@ import torch
 from .build import LIB
 
 VP_MODE_MEAN, VP_MODE_SURROGATE, VP_MODE_FULL = 0, 1, 2
-VP_WS_ROUTER, VP_WS_LAYER, VP_WS_STACK = 0, 1, 2
+VP_WS_ROUTER, VP_WS_LAYER, VP_WS_STACK, VP_WS_STACK_MERGE = 0, 1, 2, 3
 VP_ACT_NONE, VP_ACT_GELU = 0, 1
 VP_DEVERR_WAIT_TIMEOUT, VP_DEVERR_NAN_SALIENCY = 1, 2
 VP_VARIANT_MEAN_QPOOL, VP_VARIANT_MEAN_CONTEXT, VP_VARIANT_NO_RESIDUAL, VP_VARIANT_LINEAR_ATTENTION = 1, 2, 4, 8
 KERNEL_CLASSES = ["gemm", "router_pool", "router_keys", "router_r", "bin_heads", "attn_full",
-                  "surrogate", "mean", "layer_norm"]
+                  "surrogate", "mean", "layer_norm", "merge"]
 
 STATUS = {0: "VP_OK", 1: "VP_ERR_INVALID_ARG", 2: "VP_ERR_UNSUPPORTED_SHAPE", 3: "VP_ERR_ALIGNMENT",
           4: "VP_ERR_CUDA", 5: "VP_ERR_DEVICE_TIMEOUT", 6: "VP_ERR_WORKSPACE",
@@ -54,11 +54,16 @@ class VpQkOptions(Structure):
                 ("patch_start", c_int32), ("grid_w", c_int32), ("rope_base", c_float)]
 
 
+class VpMergeOptions(Structure):
+    _fields_ = [("stride", c_int32), ("tokens_per_view", c_int32), ("patch_start", c_int32),
+                ("assign_out", c_void_p)]
+
+
 class VpLayerWeights(Structure):
     _fields_ = [(n, c_void_p) for n in ("ln1_g", "ln1_b", "w_qkv", "b_qkv", "w_o", "b_o", "ls1",
                                         "ln2_g", "ln2_b", "w_fc1", "b_fc1", "w_fc2", "b_fc2", "ls2")] + \
                [("router", VpRouterWeights), ("surrogate", VpSurrogateWeights),
-                ("qk", POINTER(VpQkOptions))]
+                ("qk", POINTER(VpQkOptions)), ("merge", POINTER(VpMergeOptions))]
 
 
 _lib = None
@@ -164,7 +169,12 @@ def qk_options(w: dict = None, norm_eps: float = 1e-6, rope: bool = False, token
     return o
 
 
-def layer_weights(w: dict, qk: VpQkOptions = None) -> VpLayerWeights:
+def merge_options(stride: int, tokens_per_view: int, patch_start: int = 5, assign_out=None) -> VpMergeOptions:
+    """vp_merge_options; assign_out: int32 device tensor [N] or None."""
+    return VpMergeOptions(stride, tokens_per_view, patch_start, _p(assign_out))
+
+
+def layer_weights(w: dict, qk: VpQkOptions = None, merge: VpMergeOptions = None) -> VpLayerWeights:
     lw = VpLayerWeights(*[_p(w[k]) for k in ("ln1_g", "ln1_b", "w_qkv", "b_qkv", "w_o", "b_o", "ls1",
                                              "ln2_g", "ln2_b", "w_fc1", "b_fc1", "w_fc2", "b_fc2",
                                              "ls2")])
@@ -173,6 +183,9 @@ def layer_weights(w: dict, qk: VpQkOptions = None) -> VpLayerWeights:
     if qk is not None:
         lw.qk = ctypes.pointer(qk)
         lw._qk_keep = qk  # the struct must outlive the call
+    if merge is not None:
+        lw.merge = ctypes.pointer(merge)
+        lw._merge_keep = merge
     return lw
 
 

@@ -172,6 +172,27 @@ size_t stack_ws_bytes(const vp_dims* dm) {
          align_up(N * 4 * D * 2);
 }
 
+// Token-merging scratch (vp_merge_options): metric weights and rows, the destination and
+// membership tables, the merged tokens and their attention output.
+size_t merge_scratch_bytes(size_t N, size_t D) {
+  return align_up(64 * D * 2) + align_up(64 * sizeof(float)) + 3 * align_up(N * 64 * 2) +
+         7 * align_up((N + 1) * sizeof(int)) + 2 * align_up(N * D * 2);
+}
+
+size_t stack_merge_ws_bytes(const vp_dims* dm) {
+  const size_t N = dm->N, D = (size_t)dm->H * kHeadDim;
+  return stack_ws_bytes(dm) + merge_scratch_bytes(N, D);
+}
+
+vp_status check_merge(const vp_merge_options* mo, const vp_dims* dm) {
+  if (!mo) return VP_OK;
+  if (mo->stride < 1 || mo->tokens_per_view < 1 || mo->patch_start < 0 ||
+      mo->patch_start > mo->tokens_per_view)
+    return VP_ERR_INVALID_ARG;
+  if (dm->N % mo->tokens_per_view != 0) return VP_ERR_UNSUPPORTED_SHAPE;
+  return VP_OK;
+}
+
 // Host-side checks of vp_qk_options; *max_pos: the largest position index a token takes.
 vp_status check_qk(const vp_qk_options* qk, const vp_dims* dm, int* max_pos) {
   *max_pos = 0;
@@ -199,6 +220,7 @@ vp_status check_qk(const vp_qk_options* qk, const vp_dims* dm, int* max_pos) {
 struct QkArgs {
   const vp_qk_options* o;
   const float2* table;
+  const int32_t* tok_index;  // token of each row (merged tokens), or NULL
 };
 
 void set_qk(LinearArgs& la, const QkArgs* qk, int D) {
@@ -216,6 +238,7 @@ void set_qk(LinearArgs& la, const QkArgs* qk, int D) {
     la.tok_per_view = o.tokens_per_view;
     la.patch_start = o.patch_start;
     la.grid_w = o.grid_w;
+    la.tok_index = qk->tok_index;
   }
 }
 
@@ -391,6 +414,7 @@ vp_status vp_workspace_size(const vp_dims* dims, int32_t what, size_t* bytes) {
     case VP_WS_ROUTER: *bytes = heads_scratch_bytes(dims->H); break;
     case VP_WS_LAYER: *bytes = layer_ws_bytes(dims); break;
     case VP_WS_STACK: *bytes = stack_ws_bytes(dims); break;
+    case VP_WS_STACK_MERGE: *bytes = stack_merge_ws_bytes(dims); break;
     default: return VP_ERR_INVALID_ARG;
   }
   return VP_OK;
@@ -567,7 +591,7 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
   float2* rope = reinterpret_cast<float2*>(p);
   p += align_up(kRopeTableBytes);
   if (qk && qk->rope) VP_TRY(from_cuda(launch_rope_table(max_pos, qk->rope_base, rope, st)));
-  const QkArgs qa{qk, rope};
+  const QkArgs qa{qk, rope, nullptr};
   __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
   p += align_up(N * 3 * D * 2);
   __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p);
@@ -587,6 +611,7 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
   if (!aligned16(x_inout)) return VP_ERR_ALIGNMENT;
   const int D = dims->H * kHeadDim;
   if (!ln_width_supported(D)) return VP_ERR_UNSUPPORTED_SHAPE;
+  bool any_merge = false;
   for (int l = 0; l < n_layers; ++l) {
     const vp_layer_weights& w = layers[l];
     if (!w.ln1_g || !w.ln1_b || !w.w_qkv || !w.w_o || !w.ls1 || !w.ln2_g || !w.ln2_b ||
@@ -602,8 +627,11 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     VP_TRY(check_surrogate_weights(&w.surrogate));
     int max_pos = 0;
     VP_TRY(check_qk(w.qk, dims, &max_pos));
+    VP_TRY(check_merge(w.merge, dims));
+    any_merge = any_merge || w.merge != nullptr;
   }
-  if (!ws || ws_bytes < stack_ws_bytes(dims)) return VP_ERR_WORKSPACE;
+  if (!ws || ws_bytes < (any_merge ? stack_merge_ws_bytes(dims) : stack_ws_bytes(dims)))
+    return VP_ERR_WORKSPACE;
   VP_TRY(check_device());
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t N = dims->N;
@@ -630,14 +658,37 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
   __nv_bfloat16* qkv = reinterpret_cast<__nv_bfloat16*>(p);
   __nv_bfloat16* y = reinterpret_cast<__nv_bfloat16*>(p + align_up(N * 3 * D * 2));
   __nv_bfloat16* hid = reinterpret_cast<__nv_bfloat16*>(p);  // reuses the QKV / Y region
+  p += align_up(N * 4 * D * 2);
+  MergeScratch ms{};  // after the stack's own regions (VP_WS_STACK_MERGE)
+  if (any_merge) {
+    ms.wbar = reinterpret_cast<__nv_bfloat16*>(p);
+    p += align_up(64 * D * 2);
+    ms.bbar = reinterpret_cast<float*>(p);
+    p += align_up(64 * sizeof(float));
+    __nv_bfloat16** rows64[3] = {&ms.kbar, &ms.m, &ms.m_dst};
+    for (__nv_bfloat16** q : rows64) {
+      *q = reinterpret_cast<__nv_bfloat16*>(p);
+      p += align_up(N * 64 * 2);
+    }
+    int** ints[7] = {&ms.row_of, &ms.dst_tok, &ms.assign, &ms.cnt, &ms.offs, &ms.fill, &ms.members};
+    for (int** q : ints) {
+      *q = reinterpret_cast<int*>(p);
+      p += align_up((N + 1) * sizeof(int));
+    }
+    ms.xm = reinterpret_cast<__nv_bfloat16*>(p);
+    p += align_up(N * D * 2);
+    ms.err = sc.err;
+  }
+  __nv_bfloat16* merged_out = any_merge ? reinterpret_cast<__nv_bfloat16*>(p) : nullptr;  // [Np][D]
   __nv_bfloat16* x = reinterpret_cast<__nv_bfloat16*>(x_inout);
   const int sms = device_sm_count();
   VP_TRY(from_cuda(launch_ln_partials(dims->N, D, x, part, st)));
   for (int l = 0; l < n_layers; ++l) {
     const vp_layer_weights& w = layers[l];
-    VP_TRY(from_cuda(launch_ln_fold_weights(3 * D, D,
-                                            reinterpret_cast<const __nv_bfloat16*>(w.w_qkv),
-                                            w.ln1_g, w.ln1_b, w.b_qkv, wq, cq, bq, st)));
+    if (!w.merge)
+      VP_TRY(from_cuda(launch_ln_fold_weights(3 * D, D,
+                                              reinterpret_cast<const __nv_bfloat16*>(w.w_qkv),
+                                              w.ln1_g, w.ln1_b, w.b_qkv, wq, cq, bq, st)));
     if (w.qk && w.qk->rope &&
         !(rope_built && rope_built->rope_base == w.qk->rope_base &&
           rope_built->tokens_per_view == w.qk->tokens_per_view &&
@@ -647,16 +698,35 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
       VP_TRY(from_cuda(launch_rope_table(max_pos, w.qk->rope_base, rope, st)));
       rope_built = w.qk;
     }
-    const QkArgs qa{w.qk, rope};
-    // (1)-(3) X <- X + LS1 (Y W_O + b_O) in place, Y the routed attention of LN1(X)
-    const LnFold fold{part, cq, ln_eps};
-    VP_TRY(run_layer(dims, x, reinterpret_cast<const vp_bf16*>(wq), bq, w.w_o, w.b_o, w.ls1, x,
-                     &w.router, &w.surrogate,
-                     force_modes ? force_modes + (size_t)l * dims->H : nullptr, x, qkv, y,
-                     s_out ? s_out + (size_t)l * dims->H : nullptr,
-                     s_attn_out ? s_attn_out + (size_t)l * dims->H : nullptr,
-                     modes_out ? modes_out + (size_t)l * dims->H : nullptr, sc, st, &fold,
-                     &qa));
+    const int32_t* fm = force_modes ? force_modes + (size_t)l * dims->H : nullptr;
+    float* s_l = s_out ? s_out + (size_t)l * dims->H : nullptr;
+    float* sa_l = s_attn_out ? s_attn_out + (size_t)l * dims->H : nullptr;
+    int32_t* m_l = modes_out ? modes_out + (size_t)l * dims->H : nullptr;
+    if (w.merge) {
+      // (1) X~ = LN1(X); merge X~ (vp_merge_options); (2)-(3) routed attention of the merged
+      // tokens; unmerge: X_i += LS1 (.) A[merged row of i]
+      VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln1_g, w.ln1_b, ln_eps, zt, st)));
+      const MergeGeo g = make_merge_geo(dims->N, w.merge->tokens_per_view, w.merge->patch_start,
+                                        w.merge->stride);
+      VP_TRY(from_cuda(launch_merge_prepare(g, dims->H, zt,
+                                            reinterpret_cast<const __nv_bfloat16*>(w.w_qkv),
+                                            w.b_qkv, ms, sms, st)));
+      if (w.merge->assign_out)
+        VP_TRY(from_cuda(cudaMemcpyAsync(w.merge->assign_out, ms.assign, N * sizeof(int),
+                                         cudaMemcpyDeviceToDevice, st)));
+      vp_dims dm = *dims;
+      dm.N = g.Np;
+      const QkArgs qm{w.qk, rope, ms.dst_tok};
+      VP_TRY(run_layer(&dm, ms.xm, w.w_qkv, w.b_qkv, w.w_o, w.b_o, nullptr, nullptr, &w.router,
+                       &w.surrogate, fm, merged_out, qkv, y, s_l, sa_l, m_l, sc, st, nullptr, &qm));
+      VP_TRY(from_cuda(launch_unmerge_residual(dims->N, D, ms.assign, merged_out, w.ls1, x, st)));
+    } else {
+      const QkArgs qa{w.qk, rope, nullptr};
+      // (1)-(3) X <- X + LS1 (Y W_O + b_O) in place, Y the routed attention of LN1(X)
+      const LnFold fold{part, cq, ln_eps};
+      VP_TRY(run_layer(dims, x, reinterpret_cast<const vp_bf16*>(wq), bq, w.w_o, w.b_o, w.ls1, x,
+                       &w.router, &w.surrogate, fm, x, qkv, y, s_l, sa_l, m_l, sc, st, &fold, &qa));
+    }
     // (4) Z~ = LN2(X_attn); X <- X_attn + LS2 FFN(Z~)
     VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, zt, st)));
     LinearArgs f1{};

@@ -57,6 +57,7 @@ struct GemmParams {
   float qk_eps;
   const float2* rope_cs;
   int tok_per_view, patch_start, grid_w;
+  const int32_t* tok_index;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -300,7 +301,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float* nbv = is_q ? prm.qn_b : prm.kn_b;
         int py = 0, px = 0;  // the row's position inside its view
         if (prm.rope_cs) {
-          const int t = row % prm.tok_per_view - prm.patch_start;
+          const int tok = prm.tok_index && row_ok ? __ldg(prm.tok_index + row) : row;
+          const int t = tok % prm.tok_per_view - prm.patch_start;
           if (t >= 0) {
             py = t / prm.grid_w + 1;
             px = t - (py - 1) * prm.grid_w + 1;
@@ -503,7 +505,7 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   GemmParams prm{a.M,     a.N,   a.K,   a.bias,      a.act,  a.scale,   a.residual,
                  a.out,   a.err, a.ln_part, a.ln_c, a.ln_eps, a.part_out,
                  qk ? a.qk_cols : 0, a.qn_g, a.qn_b, a.kn_g, a.kn_b, a.qk_eps, a.rope_cs,
-                 a.tok_per_view, a.patch_start, a.grid_w};
+                 a.tok_per_view, a.patch_start, a.grid_w, a.tok_index};
   prof_before(VP_KERNEL_GEMM, st);
   gemm_kernel<<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
   prof_after(st);

@@ -147,6 +147,7 @@ struct LinearArgs {
   float qk_eps;
   const float2* rope_cs;  // NULL: no RoPE
   int tok_per_view, patch_start, grid_w;
+  const int32_t* tok_index;  // RoPE: token index of output row r (merged tokens), or NULL (r)
 };
 cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st);
 
@@ -161,6 +162,37 @@ cudaError_t launch_rope_table(int max_pos, float base, float2* table, cudaStream
 cudaError_t launch_ln_fold_weights(int Nout, int K, const __nv_bfloat16* W, const float* g,
                                    const float* beta, const float* b, __nv_bfloat16* Wp,
                                    float* c, float* bp, cudaStream_t st);
+
+// Token merging around a block's attention (merge.cu, vp_merge_options).
+struct MergeGeo {
+  int N, P, ps, stride;
+  int Dv;  // destinations per view after the first
+  int Np;  // merged tokens
+};
+MergeGeo make_merge_geo(int N, int P, int ps, int stride);
+struct MergeScratch {
+  __nv_bfloat16* wbar;   // [64][D] head-mean key weights
+  float* bbar;           // [64]
+  __nv_bfloat16* kbar;   // [N][64] metric
+  __nv_bfloat16* m;      // [N][64] unit metric
+  __nv_bfloat16* m_dst;  // [Np][64]
+  int* row_of;           // [N] merged row of a destination, -1 for sources
+  int* dst_tok;          // [Np] token of merged row
+  int* assign;           // [N] merged row every token joins
+  int* cnt;              // [Np]
+  int* offs;             // [Np + 1]
+  int* fill;             // [Np]
+  int* members;          // [N]
+  __nv_bfloat16* xm;     // [Np][D] merged tokens
+  unsigned int* err;
+};
+// x~ [N][D] -> s.assign, s.dst_tok, s.xm (D = 64 H, D % 256 == 0).
+cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* xt,
+                                 const __nv_bfloat16* w_qkv, const float* b_qkv,
+                                 const MergeScratch& s, int num_sms, cudaStream_t st);
+// x[i] += ls (.) a[assign[i]] over N rows of D channels.
+cudaError_t launch_unmerge_residual(int N, int D, const int* assign, const __nv_bfloat16* a,
+                                    const float* ls, __nv_bfloat16* x, cudaStream_t st);
 
 cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float* g,
                               const float* b, float eps, __nv_bfloat16* out, cudaStream_t st);

@@ -1,0 +1,117 @@
+"""GPU parity of token merging around a block's attention (vp_merge_options, the library's
+reading of the paper's ToMe + VGGT-Prime combination) against the float64 oracle: the
+matching (every source's destination is the most similar one, up to the metric's bf16
+resolution; exact wherever the best destination leads clearly) and, with the library's
+matching fed to the oracle, the stack output."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from tests.helpers import BF16_STEP, compare
+
+pytestmark = pytest.mark.gpu
+
+vpb = pytest.importorskip("paper_2609_23733_gb300.binding")
+
+P224 = synth.tokens_per_view(224)  # 261
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    vpb.lib()
+
+
+def _f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def _check_matching(got, info, what):
+    """got: the library's merged row per token; info: the oracle block's merge record."""
+    mg = info["merge"]
+    own, scores = mg["assign"], mg["scores"]
+    dst = np.zeros(len(own), bool)
+    dst[mg["dst_tok"]] = True
+    assert np.array_equal(got[dst], own[dst]), what  # destinations keep their own row
+    src = np.nonzero(~dst)[0]
+    best = scores[src].max(axis=1)
+    chosen = scores[src, got[src]]
+    # unit metric rows are bf16 on both sides (they may differ by an ulp): 2e-2 of cosine
+    assert np.all(chosen >= best - 2e-2), (what, float((best - chosen).max()))
+    top2 = np.sort(scores[src], axis=1)[:, -2:]
+    clear = top2[:, 1] - top2[:, 0] > 4e-2
+    assert clear.sum() >= 100, (what, int(clear.sum()))  # random metrics: about a third lead clearly
+    assert np.array_equal(got[src][clear], own[src][clear]), what
+
+
+@pytest.mark.parametrize("strides,with_qk", [((4, 10), False), ((10, 4), True)])
+def test_stack_with_token_merging(strides, with_qk):
+    """Two blocks over 4 views at 224 px (1,044 tokens), merging ~75 % (stride 4) and ~90 %
+    (stride 10) of the tokens, routed heads in every mode."""
+    N, L = 4 * P224, 2
+    g = synth.rng(21)
+    wts = [synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1) for _ in range(L)]
+    for w in wts:
+        w["ls1"] = (0.5 * w["ls1"]).astype(np.float32)
+        w["ls2"] = (0.5 * w["ls2"]).astype(np.float32)
+    qs = [synth.make_qk_norm_weights(g) for _ in range(L)]
+    x_bits = synth.make_tokens(21, N)
+    force = np.array([[2, 1, 0, 1] * 4, synth.forced_mix(16, 0.5)])
+    dm = vpb.dims(N, 16)
+    dws = [vpb.to_device(w) for w in wts]
+    dqs = [vpb.to_device(q) for q in qs]
+    assign = [torch.full((N,), -1, dtype=torch.int32, device="cuda") for _ in range(L)]
+    rope = dict(tokens_per_view=P224, patch_start=5, grid_w=16, base=100.0)
+    layers = []
+    for l in range(L):
+        qk = vpb.qk_options(dqs[l], norm_eps=1e-6, rope=True, tokens_per_view=P224, patch_start=5, grid_w=16,
+                            rope_base=100.0) if with_qk else None
+        layers.append(vpb.layer_weights(dws[l], qk, vpb.merge_options(strides[l], P224, 5, assign[l])))
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
+    x = vpb.bf16_from_bits(x_bits)
+    modes = torch.zeros(L, 16, dtype=torch.int32, device="cuda")
+    s = torch.zeros(L, 16, device="cuda")
+    vpb.vp_global_stack(dm, x, layers, torch.tensor(force, dtype=torch.int32, device="cuda"), modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    got_assign = [a.cpu().numpy().astype(np.int64) for a in assign]
+    merge = [{"stride": st, "tokens_per_view": P224, "patch_start": 5} for st in strides]
+    qk = None
+    if with_qk:
+        qk = [{"q_norm": (q["q_norm_g"], q["q_norm_b"]), "k_norm": (q["k_norm_g"], q["k_norm_b"]), "eps": 1e-6,
+               "rope": rope} for q in qs]
+    want, infos = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w) for w in wts],
+                                      force_modes=force, qk=qk, merge=merge, assign=got_assign)
+    for l in range(L):
+        _check_matching(got_assign[l], infos[l], f"block {l}")
+        # the first view stays whole; later views keep 5 special tokens and every stride-th patch
+        assert len(infos[l]["merge"]["dst_tok"]) == P224 + 3 * (5 + -(-256 // strides[l]))
+    np.testing.assert_array_equal(modes.cpu().numpy(), force)
+    compare(_f64(x), want, rel=L * BF16_STEP, what="2-block stack with token merging")
+
+
+def test_merge_options_are_validated():
+    N = 4 * P224
+    g = synth.rng(22)
+    dw = vpb.to_device(synth.make_layer_weights(g, block=True))
+    x = torch.zeros(N, 1024, dtype=torch.bfloat16, device="cuda")
+    modes = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
+    s = torch.zeros(1, 16, device="cuda")
+    dm = vpb.dims(N, 16)
+    small = vpb.workspace(dm, vpb.VP_WS_STACK)  # no room for the merging scratch
+    with pytest.raises(vpb.VPError) as e:
+        vpb.vp_global_stack(dm, x, [vpb.layer_weights(dw, None, vpb.merge_options(4, P224, 5))], None, modes,
+                            s, 1e-6, small)
+    assert e.value.status == 6
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
+    with pytest.raises(vpb.VPError) as e:  # views of 300 tokens do not tile N
+        vpb.vp_global_stack(dm, x, [vpb.layer_weights(dw, None, vpb.merge_options(4, 300, 5))], None, modes, s,
+                            1e-6, ws)
+    assert e.value.status == 2
+    with pytest.raises(vpb.VPError) as e:
+        vpb.vp_global_stack(dm, x, [vpb.layer_weights(dw, None, vpb.merge_options(0, P224, 5))], None, modes, s,
+                            1e-6, ws)
+    assert e.value.status == 1
