@@ -10,9 +10,8 @@
 //   merge: a merged token is the mean of its destination and the sources that joined it;
 //   unmerge: every token takes its merged token's attention output.
 // Kernels: the head-mean key weights, the metric GEMM (gemm_kernel), unit metric rows and the
-// destination table, the matching (mma.sync tiles of 16 sources x 64 destinations with a
-// running argmax; the max of a thread's 16 scores is taken first and the index searched only
-// when it improves), counting / scan / fill of each merged token's members, their mean, and
+// destination table, the matching (tcgen05 scores of 128 sources x 256 destinations per MMA
+// group with a running argmax in the epilogue), counting / scan / fill of each merged token's members, their mean, and
 // the unmerge fused with LayerScale and the residual add.
 #include <math.h>
 
@@ -22,15 +21,6 @@
 namespace vp {
 
 namespace {
-
-// D (16 x 8, fp32) += A (16 x 16, bf16, row) B (16 x 8, bf16, col): one warp, mma.sync.
-__device__ __forceinline__ void mma16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 
 // Destination test and merged row of token i (MergeGeo: views of P tokens, ps special tokens,
 // every stride-th patch of views 1.. is a destination, Dv destinations per such view).
@@ -83,94 +73,238 @@ __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_b
   }
 }
 
-constexpr int kMatchWarps = 8;     // 16 source rows per warp
-constexpr int kMatchDst = 64;      // destinations per shared-memory tile
-constexpr int kMatchStride = 72;   // padded bf16 row: conflict-free fragment loads
+// Matching on the tensor cores: scores S = M_src M_dst^T (cosines of unit keys) for 128 source
+// rows at a time against chunks of 256 destinations, with a running argmax over the chunks.
+// Persistent CTAs (one per SM) take source tiles t = blockIdx.x, + gridDim.x, ...
+//   warp 0      TMA: the tile's 128 source rows once (16 KB), destination chunks (256 rows x
+//               64 channels, 32 KB, 128-byte swizzle) through a kMatchStages ring;
+//   warp 1      TMEM owner and MMA issue: four tcgen05.mma M128 N256 K16 per chunk into one
+//               of two 256-column fp32 accumulators (the epilogue of one chunk overlaps the
+//               MMAs of the next);
+//   warps 4-19  argmax: a source row (TMEM lane) and a quarter of each chunk's columns per
+//               thread, 32 columns per tcgen05.ld (the next in flight), the max of the 32 by
+//               a tree first and the column only when it reaches the row's best (equal
+//               scores go to the lower index); the four parts combine at the end of the tile.
+constexpr int kMatchStages = 6;
+constexpr int kMatchN = 256;
+constexpr int kMatchParts = 4;  // column parts of a chunk (argmax warps per TMEM lane quarter)
+constexpr int kMatchThreads = 128 + 128 * kMatchParts;
+constexpr uint32_t kMatchTmemCols = 512;
 
-// assign[i] = merged row of token i's destination: its own for destinations, the argmax of
-// the cosine similarity over all destinations for sources.
-__global__ void __launch_bounds__(32 * kMatchWarps) tome_match_kernel(
-    MergeGeo g, const __nv_bfloat16* m, const __nv_bfloat16* m_dst, const int* row_of,
-    int* assign) {
-  __shared__ __align__(16) __nv_bfloat16 sd[kMatchDst * kMatchStride];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int gq = lane >> 2, tq = lane & 3;
-  const int r0 = (blockIdx.x * kMatchWarps + warp) * 16;  // this warp's 16 source rows
-  // A fragments (16 rows x 64 channels), kept in registers for the whole sweep.
-  uint32_t af[4][4];
-  {
-    const int ra = min(r0 + gq, g.N - 1), rb = min(r0 + gq + 8, g.N - 1);
-    const uint32_t* pa = reinterpret_cast<const uint32_t*>(m + (size_t)ra * 64);
-    const uint32_t* pb = reinterpret_cast<const uint32_t*>(m + (size_t)rb * 64);
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      af[kk][0] = __ldg(pa + 8 * kk + tq);
-      af[kk][1] = __ldg(pb + 8 * kk + tq);
-      af[kk][2] = __ldg(pa + 8 * kk + tq + 4);
-      af[kk][3] = __ldg(pb + 8 * kk + tq + 4);
+struct MatchSmem {
+  __nv_bfloat16 src[128 * 64];
+  __nv_bfloat16 dst[kMatchStages][kMatchN * 64];
+  uint64_t src_full, src_empty;
+  uint64_t dst_full[kMatchStages], dst_empty[kMatchStages];
+  uint64_t acc_full[2], acc_empty[2], drain;
+  uint64_t part_post, part_taken;  // parts 1.. posted their best / part 0 read them
+  float part_v[kMatchParts - 1][128];  // parts 1..'s best per row, for the combine
+  int part_i[kMatchParts - 1][128];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__global__ void __launch_bounds__(kMatchThreads, 1)
+    tome_match_kernel(const __grid_constant__ CUtensorMap tmap_src,
+                      const __grid_constant__ CUtensorMap tmap_dst, MergeGeo g, const int* row_of,
+                      int* assign, unsigned int* err) {
+  extern __shared__ unsigned char smem_raw[];
+  MatchSmem& sm = *reinterpret_cast<MatchSmem*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int n_tiles = (g.N + 127) / 128;
+  const int n_chunks = (g.Np + kMatchN - 1) / kMatchN;
+  if ((int)blockIdx.x >= n_tiles) return;
+  // The CTAs sweep the destination chunks from staggered starts, so that they do not all
+  // read the same chunk (the same L2 lines) at the same time.
+  const int ch_start = (int)(((long long)blockIdx.x * n_chunks) / gridDim.x);
+  const int warp = warp_uniform_id(), lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.src_full, 1);
+    mbar_init(&sm.src_empty, 1);
+    for (int s = 0; s < kMatchStages; ++s) {
+      mbar_init(&sm.dst_full[s], 1);
+      mbar_init(&sm.dst_empty[s], 1);
     }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.acc_full[b], 1);
+      mbar_init(&sm.acc_empty[b], 128 * kMatchParts);
+    }
+    mbar_init(&sm.drain, 1);
+    mbar_init(&sm.part_post, 128 * (kMatchParts - 1));
+    mbar_init(&sm.part_taken, 128);
+    sm.abort_flag = 0;
+    fence_mbarrier_init();
+    fence_proxy_async_smem();
+    tma_prefetch_desc(&tmap_src);
+    tma_prefetch_desc(&tmap_dst);
   }
-  float bv0 = -INFINITY, bv1 = -INFINITY;
-  int bi0 = 0, bi1 = 0;  // a valid row even if no score compares (NaN metric)
-  for (int n0 = 0; n0 < g.Np; n0 += kMatchDst) {
-    __syncthreads();  // the previous tile is no longer read
-    for (int q = threadIdx.x; q < kMatchDst * 8; q += blockDim.x) {  // 16-byte pieces
-      const int rr = q >> 3, cc = q & 7;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (n0 + rr < g.Np) v = __ldg(reinterpret_cast<const uint4*>(m_dst + (size_t)(n0 + rr) * 64) + cc);
-      *reinterpret_cast<uint4*>(&sd[rr * kMatchStride + cc * 8]) = v;
-    }
-    __syncthreads();
-    float c[8][4];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      c[j][0] = c[j][1] = c[j][2] = c[j][3] = 0.f;
-      const uint32_t* brow = reinterpret_cast<const uint32_t*>(&sd[(8 * j + gq) * kMatchStride]);
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk)
-        mma16816(c[j], af[kk], brow[8 * kk + tq], brow[8 * kk + tq + 4]);
-      if (n0 + 8 * j + 2 * tq >= g.Np) c[j][0] = c[j][2] = -INFINITY;
-      if (n0 + 8 * j + 2 * tq + 1 >= g.Np) c[j][1] = c[j][3] = -INFINITY;
-    }
-    float m0 = c[0][0], m1 = c[0][2];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      m0 = fmax3(m0, c[j][0], c[j][1]);
-      m1 = fmax3(m1, c[j][2], c[j][3]);
-    }
-    if (m0 > bv0) {  // first column (lowest index) holding the new maximum
-      int best = 0x7fffffff;
-#pragma unroll
-      for (int j = 7; j >= 0; --j) {
-        if (c[j][1] == m0) best = n0 + 8 * j + 2 * tq + 1;
-        if (c[j][0] == m0) best = n0 + 8 * j + 2 * tq;
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, kMatchTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    uint32_t lc = 0, ic = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ic) {
+      ok = mbar_wait_warp(&sm.src_empty, (ic & 1) ^ 1, err, abort_flag);
+      if (!ok) break;
+      if (elect_one()) {
+        mbar_arrive_expect_tx(&sm.src_full, 128 * 64 * 2);
+        tma_load_2d(sm.src, &tmap_src, &sm.src_full, 0, t * 128);
       }
-      bv0 = m0;
-      bi0 = best;
-    }
-    if (m1 > bv1) {
-      int best = 0x7fffffff;
-#pragma unroll
-      for (int j = 7; j >= 0; --j) {
-        if (c[j][3] == m1) best = n0 + 8 * j + 2 * tq + 1;
-        if (c[j][2] == m1) best = n0 + 8 * j + 2 * tq;
+      __syncwarp();
+      for (int ch = 0; ch < n_chunks; ++ch, ++lc) {
+        const int st = lc % kMatchStages;
+        ok = mbar_wait_warp(&sm.dst_empty[st], ((lc / kMatchStages) & 1) ^ 1, err, abort_flag);
+        if (!ok) break;
+        if (elect_one()) {
+          const int chunk = (ch_start + ch) % n_chunks;
+          mbar_arrive_expect_tx(&sm.dst_full[st], kMatchN * 64 * 2);
+          tma_load_2d(sm.dst[st], &tmap_dst, &sm.dst_full[st], 0, chunk * kMatchN);
+        }
+        __syncwarp();
       }
-      bv1 = m1;
-      bi1 = best;
+    }
+    if (!ok && lane == 0) {  // let issued copies land before the CTA releases its smem
+      if (ic > 0)
+        for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.src_full, (ic - 1) & 1); ++k) {}
+      for (int s = 0; s < kMatchStages; ++s) {
+        if (lc > (uint32_t)s) {
+          const uint32_t last = (lc - 1 - s) / kMatchStages * kMatchStages + s;
+          for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.dst_full[s], (last / kMatchStages) & 1); ++k) {}
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issue
+    const uint32_t idesc = idesc_bf16(128, kMatchN, 0, 0);
+    const uint64_t da = sdesc_sw128(smem_u32(sm.src));
+    uint32_t lc = 0, ic = 0, ac = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ic) {
+      ok = mbar_wait_warp(&sm.src_full, ic & 1, err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      for (int ch = 0; ch < n_chunks; ++ch, ++lc, ++ac) {
+        const int st = lc % kMatchStages;
+        const uint32_t ab = ac & 1;
+        ok = mbar_wait_warp(&sm.dst_full[st], (lc / kMatchStages) & 1, err, abort_flag) &&
+             mbar_wait_warp(&sm.acc_empty[ab], ((ac >> 1) & 1) ^ 1, err, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        const uint64_t db = sdesc_sw128(smem_u32(sm.dst[st]));
+        if (elect_one()) {
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // K = 64 channels: 4 x K16, +32 bytes per step
+            tc_mma_ss(tmem + ab * kMatchN, da + 2 * kk, db + 2 * kk, idesc, kk > 0 ? 1u : 0u);
+          tc_commit(&sm.acc_full[ab]);
+          tc_commit(&sm.dst_empty[st]);
+          if (ch == n_chunks - 1) tc_commit(&sm.src_empty);
+        }
+        __syncwarp();
+      }
+    }
+    if (!ok) {
+      if (elect_one()) {
+        tc_commit(&sm.drain);
+        for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.drain, 0); ++k) {}
+      }
+      __syncwarp();
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------ running argmax
+    constexpr int kCols = kMatchN / kMatchParts;  // columns of a part
+    const int quarter = warp & 3, part = (warp - 4) >> 2;
+    const int rit = quarter * 32 + lane;  // row in the tile
+    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16) + part * kCols;
+    uint32_t ac = 0, ic = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ic) {
+      float bv = -INFINITY;
+      int bi = 0x7fffffff;
+      for (int ch = 0; ch < n_chunks; ++ch, ++ac) {
+        const uint32_t ab = ac & 1;
+        ok = mbar_wait_warp(&sm.acc_full[ab], (ac >> 1) & 1, err, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        const int c0 = ((ch_start + ch) % n_chunks) * kMatchN + part * kCols;  // first destination
+        const int valid = g.Np - c0;                         // columns past it hold no destination
+        float v[2][32];
+        tmem_ld32(t_lane + ab * kMatchN, v[0]);
+        tmem_wait_ld();
+#pragma unroll
+        for (int p = 0; p < kCols / 32; ++p) {
+          if (p + 1 < kCols / 32) tmem_ld32(t_lane + ab * kMatchN + 32 * (p + 1), v[(p + 1) & 1]);
+          float* x = v[p & 1];
+          if (32 * p + 32 > valid) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k)
+              if (32 * p + k >= valid) x[k] = -INFINITY;
+          }
+          float q[4];  // four independent max chains, then a short tree
+#pragma unroll
+          for (int k = 0; k < 4; ++k) q[k] = fmaxf(x[k], x[k + 4]);
+#pragma unroll
+          for (int k = 8; k < 32; k += 8)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) q[e] = fmaxf(q[e], x[k + e]), q[e] = fmaxf(q[e], x[k + 4 + e]);
+          const float mx = fmaxf(fmaxf(q[0], q[1]), fmaxf(q[2], q[3]));
+          if (mx >= bv) {  // chunks come in rotated order: equal scores go to the lower index
+            int best = 0;
+#pragma unroll
+            for (int k = 31; k >= 0; --k)
+              if (x[k] == mx) best = c0 + 32 * p + k;
+            if (mx > bv || best < bi) {
+              bv = mx;
+              bi = best;
+            }
+          }
+          tmem_wait_ld();
+        }
+        tc_fence_before();
+        mbar_arrive(&sm.acc_empty[ab]);
+      }
+      if (!ok) break;
+      // Combine the parts through shared memory and two mbarriers (bounded waits): parts 1..
+      // post their best once part 0 has read the previous tile's; part 0 decides (larger
+      // score, then lower index).
+      if (part > 0) {
+        ok = mbar_wait_warp(&sm.part_taken, (ic & 1) ^ 1, err, abort_flag);
+        if (!ok) break;
+        sm.part_v[part - 1][rit] = bv;
+        sm.part_i[part - 1][rit] = bi;
+        mbar_arrive(&sm.part_post);
+      } else {
+        ok = mbar_wait_warp(&sm.part_post, ic & 1, err, abort_flag);
+        if (!ok) break;
+#pragma unroll
+        for (int q = 0; q < kMatchParts - 1; ++q) {
+          const float ov = sm.part_v[q][rit];
+          const int oi = sm.part_i[q][rit];
+          if (ov > bv || (ov == bv && oi < bi)) {
+            bv = ov;
+            bi = oi;
+          }
+        }
+        mbar_arrive(&sm.part_taken);
+        const int row = t * 128 + rit;
+        if (bi >= g.Np) bi = 0;  // no score compared (NaN metric): any valid row
+        if (row < g.N) assign[row] = row_of[row] >= 0 ? row_of[row] : bi;
+      }
     }
   }
-  // Across the four threads of a row: larger score, then lower index.
-#pragma unroll
-  for (int o = 1; o < 4; o <<= 1) {
-    const float v0 = __shfl_xor_sync(0xffffffffu, bv0, o), v1 = __shfl_xor_sync(0xffffffffu, bv1, o);
-    const int i0 = __shfl_xor_sync(0xffffffffu, bi0, o), i1 = __shfl_xor_sync(0xffffffffu, bi1, o);
-    if (v0 > bv0 || (v0 == bv0 && i0 < bi0)) { bv0 = v0; bi0 = i0; }
-    if (v1 > bv1 || (v1 == bv1 && i1 < bi1)) { bv1 = v1; bi1 = i1; }
-  }
-  if (tq == 0) {
-    const int ra = r0 + gq, rb = r0 + gq + 8;
-    if (ra < g.N) assign[ra] = row_of[ra] >= 0 ? row_of[ra] : bi0;
-    if (rb < g.N) assign[rb] = row_of[rb] >= 0 ? row_of[rb] : bi1;
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kMatchTmemCols);
   }
 }
 
@@ -215,7 +349,7 @@ __global__ void merge_fill_kernel(int N, const int* assign, const int* offs, int
 // One warp per merged token: the fp32 mean of its members' rows of x~ (D = 256 C; lane l
 // holds 16-byte chunks c 32 + l).
 template <int C>
-__global__ void merge_mean_kernel(int Np, const __nv_bfloat16* xt, const int* offs,
+__global__ void __launch_bounds__(256, C <= 4 ? 3 : 1) merge_mean_kernel(int Np, const __nv_bfloat16* xt, const int* offs,
                                   const int* members, __nv_bfloat16* xm) {
   constexpr int D = 256 * C;
   const int lane = threadIdx.x & 31;
@@ -227,17 +361,31 @@ __global__ void merge_mean_kernel(int Np, const __nv_bfloat16* xt, const int* of
   for (int c = 0; c < C; ++c)
 #pragma unroll
     for (int k = 0; k < 8; ++k) acc[c][k] = 0.f;
-  for (int q = b; q < e; ++q) {
-    const int i = members[q];
+  // Member indices 32 at a time (one coalesced load), then their rows, two in flight.
+  for (int q0 = b; q0 < e; q0 += 32) {
+    const int mine = q0 + lane < e ? members[q0 + lane] : 0;
+    const int nm = min(32, e - q0);
+    for (int k = 0; k < nm; k += 2) {  // two rows' loads issued before any arithmetic
+      uint4 u[2][C];
 #pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint4 u = __ldg(reinterpret_cast<const uint4*>(xt + (size_t)i * D + (c * 32 + lane) * 8));
-      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+      for (int j = 0; j < 2; ++j) {
+        const int i = __shfl_sync(0xffffffffu, mine, min(k + j, nm - 1));
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        acc[c][2 * k] += bf16_lo(w[k]);
-        acc[c][2 * k + 1] += bf16_hi(w[k]);
+        for (int c = 0; c < C; ++c)
+          u[j][c] = k + j < nm ? __ldg(reinterpret_cast<const uint4*>(xt + (size_t)i * D + (c * 32 + lane) * 8))
+                               : make_uint4(0u, 0u, 0u, 0u);
       }
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t w[4] = {u[j][c].x, u[j][c].y, u[j][c].z, u[j][c].w};
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            acc[c][2 * kk] += bf16_lo(w[kk]);
+            acc[c][2 * kk + 1] += bf16_hi(w[kk]);
+          }
+        }
     }
   }
   const float inv = 1.f / (float)(e - b);
@@ -320,9 +468,17 @@ cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* 
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  CUtensorMap tsrc, tdst;  // unit metric rows, 64 channels (128 bytes), 128-byte swizzle
+  if ((e = make_tmap_bf16_2d(&tsrc, s.m, 64, (uint64_t)g.N, 64, 64, 128)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16_2d(&tdst, s.m_dst, 64, (uint64_t)g.Np, 64, 64, kMatchN)) != cudaSuccess)
+    return e;
+  const int smem = (int)sizeof(MatchSmem) + 1024;
+  if ((e = cudaFuncSetAttribute(tome_match_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                smem)) != cudaSuccess)
+    return e;
   prof_before(VP_KERNEL_MERGE, st);
-  tome_match_kernel<<<(g.N + 16 * kMatchWarps - 1) / (16 * kMatchWarps), 32 * kMatchWarps, 0, st>>>(
-      g, s.m, s.m_dst, s.row_of, s.assign);
+  tome_match_kernel<<<min(num_sms, (g.N + 127) / 128), kMatchThreads, smem, st>>>(
+      tsrc, tdst, g, s.row_of, s.assign, s.err);
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
