@@ -85,7 +85,7 @@ __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_b
 //               thread, 32 columns per tcgen05.ld (the next in flight), the max of the 32 by
 //               a tree first and the column only when it reaches the row's best (equal
 //               scores go to the lower index); the four parts combine at the end of the tile.
-constexpr int kMatchStages = 6;
+constexpr int kMatchStages = 4;
 constexpr int kMatchN = 256;
 constexpr int kMatchParts = 4;  // column parts of a chunk (argmax warps per TMEM lane quarter)
 constexpr int kMatchThreads = 128 + 128 * kMatchParts;
