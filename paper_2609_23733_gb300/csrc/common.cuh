@@ -80,12 +80,17 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned int* err,
                                           volatile int* abort_flag) {
   if (mbar_test_wait(bar, parity)) return true;  // already complete: no suspension
-  unsigned long long t0 = global_timer_ns();
+  // The time limit runs from the first check (after 255 unsuccessful tries), so that the
+  // common short wait reads no clock.
+  unsigned long long t0 = 0;
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 255u) == 0) {
       if (*abort_flag) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
+      const unsigned long long now = global_timer_ns();
+      if (t0 == 0) {
+        t0 = now;
+      } else if (now - t0 > kWaitLimitNs) {
         atomicOr(err, VP_DEVERR_WAIT_TIMEOUT);
         *abort_flag = 1;
         return false;
