@@ -623,6 +623,19 @@ def kernel_case(args):
         z = torch.zeros(H, d, device=dev)
         for _ in range(args.case_launches):
             vpb.vp_head_attention(dm, qkv, ids, off, z, z, vpb.surrogate_weights(w), y, ws)
+    elif args.kernel_case == "merge":  # one block with token merging (stride 10) over whole views
+        P = synth.tokens_per_view(518)
+        Nm = max(1, N // P) * P
+        w = vpb.to_device(synth.make_layer_weights(synth.rng(0), block=True), dev)
+        dm = vpb.dims(Nm, H)
+        ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE, dev)
+        x = torch.randn(Nm, D, device=dev).to(torch.bfloat16)
+        layer = [vpb.layer_weights(w, None, vpb.merge_options(10, P, 5))]
+        fm = torch.tensor([synth.forced_mix(H, 0.25)], dtype=torch.int32, device=dev)
+        modes = torch.zeros(1, H, dtype=torch.int32, device=dev)
+        s = torch.zeros(1, H, device=dev)
+        for _ in range(args.case_launches):
+            vpb.vp_global_stack(dm, x, layer, fm, modes, s, 1e-6, ws)
     elif args.kernel_case == "gemm_fc1":  # FFN up-projection with the GELU epilogue
         x = torch.randn(N, D, device=dev).to(torch.bfloat16)
         w1 = (torch.rand(4 * D, D, device=dev) * 0.1 - 0.05).to(torch.bfloat16)
@@ -682,7 +695,7 @@ def main():
     ap.add_argument("--no-qk", dest="qk", action="store_false")
     ap.add_argument("--no-tome", dest="tome", action="store_false")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
-                                              "surrogate", "mean", "bin"],
+                                              "surrogate", "mean", "bin", "merge"],
                     default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
     ap.add_argument("--case-tokens", type=int, default=32768)
