@@ -94,20 +94,34 @@ struct FullParams {
 
 // The work of one launch: G groups (head, kChains query tiles) over P persistent CTAs.  The
 // first R = floor(G / P) rounds take whole groups; the T = G - R P groups of the last round
-// are split along the keys into S = floor(P / T) parts (at most the number of key tiles),
-// so that T S <= P CTAs share that round instead of T.  Unit u < R P is group u; unit
-// R P + S t + s is part s of group R P + t.
+// are split along the keys into S parts each (at most the number of key tiles), T S part
+// units that the P CTAs take round-robin, so the last round lasts ceil(T S / P) parts of a
+// group instead of one whole group on T CTAs.  S minimises ceil(T S / P) (1 / S + c) with c
+// the cost of a part beyond its share of the keys (its Q load, pipeline fill and drain, and
+// the combine), taken as 1 % of a group.  Unit u < R P is group u; unit R P + S t + s is part
+// s of group R P + t.
 struct Plan {
   int R, T, S, units, whole;  // whole: units that are whole groups (they come first)
 };
+
+constexpr int kMaxParts = 64;
+constexpr float kPartCost = 0.01f;
 
 __device__ __forceinline__ Plan make_plan(int G, int P, int n_kv) {
   Plan pl;
   pl.R = G / P;
   pl.T = G - pl.R * P;
-  pl.S = pl.T > 0 ? P / pl.T : 1;
-  if (pl.S > n_kv) pl.S = n_kv;
-  if (pl.S < 2 || pl.T * pl.S > kFaTailUnits) pl.S = 1;
+  pl.S = 1;
+  if (pl.T > 0) {
+    float best = 1.f;  // S = 1: the T groups whole, one round
+    for (int S = 2; S <= kMaxParts && S <= n_kv && pl.T * S <= kFaTailUnits; ++S) {
+      const float cost = (float)((pl.T * S + P - 1) / P) * (1.f / (float)S + kPartCost);
+      if (cost < best - 1e-6f) {
+        best = cost;
+        pl.S = S;
+      }
+    }
+  }
   pl.units = pl.S == 1 ? G : pl.R * P + pl.T * pl.S;
   pl.whole = pl.S == 1 ? G : pl.R * P;
   return pl;
@@ -244,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Plan plan = make_plan(n_heads * n_groups, P, n_kv);
   // Units of this CTA: [u_begin, u_end) in steps of P.
   const int u_begin = kParts ? plan.whole + (int)blockIdx.x : (int)blockIdx.x;
-  const int u_end = kParts ? (u_begin < plan.units ? u_begin + 1 : u_begin) : plan.whole;
+  const int u_end = kParts ? plan.units : plan.whole;
   if (u_begin >= u_end) {  // uniform across the CTA
     // The parts grid completes only after the whole-group grid (its prerequisite): work
     // queued behind it then sees every row of Y.

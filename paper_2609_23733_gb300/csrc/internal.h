@@ -44,7 +44,7 @@ struct RouterScratch {
 // Full attention splits the work items of its last, partial round along the keys over the
 // CTAs that would otherwise idle; the partial results need this much scratch (units = groups
 // x splits of that round, at most one per CTA).
-constexpr int kFaTailUnits = 256;
+constexpr int kFaTailUnits = 512;
 constexpr size_t kFaPartFloats = (size_t)kFaTailUnits * 4 * 128 * 64;
 constexpr size_t kFaStatsFloats = (size_t)kFaTailUnits * 4 * 128 * 4;
 constexpr size_t kFaCountWords = (size_t)kFaTailUnits * 4 * 4;

@@ -248,14 +248,14 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
             for (int k = 0; k < 32; ++k)
               if (32 * p + k >= valid) x[k] = -INFINITY;
           }
-          float q[4];  // four independent max chains, then a short tree
+          float q[4];  // four independent 3-input max chains, then a short tree
 #pragma unroll
           for (int k = 0; k < 4; ++k) q[k] = fmaxf(x[k], x[k + 4]);
 #pragma unroll
           for (int k = 8; k < 32; k += 8)
 #pragma unroll
-            for (int e = 0; e < 4; ++e) q[e] = fmaxf(q[e], x[k + e]), q[e] = fmaxf(q[e], x[k + 4 + e]);
-          const float mx = fmaxf(fmaxf(q[0], q[1]), fmaxf(q[2], q[3]));
+            for (int e = 0; e < 4; ++e) q[e] = fmax3(q[e], x[k + e], x[k + 4 + e]);
+          const float mx = fmax3(q[0], q[1], fmaxf(q[2], q[3]));
           if (mx >= bv) {  // chunks come in rotated order: equal scores go to the lower index
             int best = 0;
 #pragma unroll
