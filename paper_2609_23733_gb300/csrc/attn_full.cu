@@ -98,14 +98,15 @@ struct FullParams {
 // units that the P CTAs take round-robin, so the last round lasts ceil(T S / P) parts of a
 // group instead of one whole group on T CTAs.  S minimises ceil(T S / P) (1 / S + c) with c
 // the cost of a part beyond its share of the keys (its Q load, pipeline fill and drain, and
-// the combine), taken as 1 % of a group.  Unit u < R P is group u; unit R P + S t + s is part
+// the combine), taken as 3 % of a group (0, 1, 3 and 6 % measured within 1 ms of each
+// other on the S = 100 stack, 0 the slowest).  Unit u < R P is group u; unit R P + S t + s is part
 // s of group R P + t.
 struct Plan {
   int R, T, S, units, whole;  // whole: units that are whole groups (they come first)
 };
 
 constexpr int kMaxParts = 64;
-constexpr float kPartCost = 0.01f;
+constexpr float kPartCost = 0.03f;
 
 __device__ __forceinline__ Plan make_plan(int G, int P, int n_kv) {
   Plan pl;
