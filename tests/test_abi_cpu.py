@@ -108,3 +108,61 @@ def test_valid_call_without_a_gpu_reports_the_device(vp):
     st = lib.vp_router(ctypes.byref(vp.dims(300)), A, ctypes.byref(rw), None, A, A, None, None, None, None,
                        A, 1 << 30, None)
     assert st == 7  # VP_ERR_UNSUPPORTED_DEVICE: nothing was enqueued
+
+
+def _fake_layer(vp, A, qk=None, merge=None):
+    lw = vp.VpLayerWeights(*([A] * 14))
+    lw.router = vp.VpRouterWeights(A, A, A, None, None, None)
+    lw.surrogate = vp.VpSurrogateWeights(*([A] * 8))
+    if qk is not None:
+        lw.qk = ctypes.pointer(qk)
+        lw._keep_qk = qk
+    if merge is not None:
+        lw.merge = ctypes.pointer(merge)
+        lw._keep_merge = merge
+    return lw
+
+
+def test_stack_options_validated_on_the_host(vp):
+    """vp_qk_options and vp_merge_options are checked before the workspace and the device:
+    the expected status comes back without a GPU."""
+    lib = vp.lib()
+    A = 0x10000
+    P = 261
+    dm = vp.dims(4 * P)
+    big = 1 << 40
+
+    def stack(lw, n_tokens=4 * P):
+        d = vp.dims(n_tokens)
+        arr = (vp.VpLayerWeights * 1)(lw)
+        return lib.vp_global_stack(ctypes.byref(d), 1, A, arr, None, None, None, None, ctypes.c_float(1e-6), A,
+                                   big, None)
+
+    # qk-norm: a scale without a shift
+    half = vp.VpQkOptions(A, None, None, None, 1e-6, 0, 1, 0, 1, 100.0)
+    assert stack(_fake_layer(vp, A, qk=half)) == 1
+    # misaligned norm parameters
+    mis = vp.VpQkOptions(A + 4, A, None, None, 1e-6, 0, 1, 0, 1, 100.0)
+    assert stack(_fake_layer(vp, A, qk=mis)) == 3
+    # RoPE: views that do not tile N, a zero-width grid, positions past the table
+    assert stack(_fake_layer(vp, A, qk=vp.VpQkOptions(None, None, None, None, 1e-6, 1, 300, 5, 16, 100.0))) == 2
+    assert stack(_fake_layer(vp, A, qk=vp.VpQkOptions(None, None, None, None, 1e-6, 1, P, 5, 0, 100.0))) == 1
+    assert stack(_fake_layer(vp, A, qk=vp.VpQkOptions(None, None, None, None, 1e-6, 1, 4096, 0, 2, 100.0)),
+                 n_tokens=4096) == 2
+    # merging: stride 0, views that do not tile N, more special tokens than a view holds
+    assert stack(_fake_layer(vp, A, merge=vp.VpMergeOptions(0, P, 5, None))) == 1
+    assert stack(_fake_layer(vp, A, merge=vp.VpMergeOptions(4, 300, 5, None))) == 2
+    assert stack(_fake_layer(vp, A, merge=vp.VpMergeOptions(4, P, P + 1, None))) == 1
+    # merging needs the larger workspace kind
+    need = vp.vp_workspace_size(dm, vp.VP_WS_STACK_MERGE)
+    assert need > vp.vp_workspace_size(dm, vp.VP_WS_STACK)
+    arr = (vp.VpLayerWeights * 1)(_fake_layer(vp, A, merge=vp.VpMergeOptions(4, P, 5, None)))
+    assert lib.vp_global_stack(ctypes.byref(dm), 1, A, arr, None, None, None, None, ctypes.c_float(1e-6), A,
+                               vp.vp_workspace_size(dm, vp.VP_WS_STACK), None) == 6
+
+
+def test_option_struct_layouts(vp):
+    # field order and sizes of the C structs (vp.h)
+    assert ctypes.sizeof(vp.VpQkOptions) == 4 * 8 + 4 + 4 * 4 + 4
+    assert ctypes.sizeof(vp.VpMergeOptions) == 3 * 4 + 4 + 8
+    assert ctypes.sizeof(vp.VpLayerWeights) == 14 * 8 + 6 * 8 + 8 * 8 + 2 * 8

@@ -115,3 +115,27 @@ def test_merge_options_are_validated():
         vpb.vp_global_stack(dm, x, [vpb.layer_weights(dw, None, vpb.merge_options(0, P224, 5))], None, modes, s,
                             1e-6, ws)
     assert e.value.status == 1
+
+
+def test_single_view_merges_nothing():
+    """One view: every token belongs to the first view, so every token is its own destination
+    (the identity matching) and the block is the unmerged block."""
+    N = P224
+    g = synth.rng(23)
+    w = synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1)
+    x_bits = synth.make_tokens(23, N)
+    force = np.array([[2, 1, 0, 1] * 4])
+    dm = vpb.dims(N, 16)
+    assign = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    layers = [vpb.layer_weights(vpb.to_device(w), None, vpb.merge_options(4, P224, 5, assign))]
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
+    x = vpb.bf16_from_bits(x_bits)
+    modes = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
+    s = torch.zeros(1, 16, device="cuda")
+    vpb.vp_global_stack(dm, x, layers, torch.tensor(force, dtype=torch.int32, device="cuda"), modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    np.testing.assert_array_equal(assign.cpu().numpy(), np.arange(N))
+    want, _ = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w)], force_modes=force,
+                                  merge=[{"stride": 4, "tokens_per_view": P224, "patch_start": 5}])
+    compare(_f64(x), want, rel=BF16_STEP, what="single view with merging on")
