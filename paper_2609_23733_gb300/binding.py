@@ -144,14 +144,24 @@ def dims(N, H=16, d=64, L=64, tau_low=0.01, tau_high=0.20, variant=0) -> VpDims:
     return VpDims(int(N), int(H), int(d), int(L), float(tau_low), float(tau_high), int(variant))
 
 
+# The weight and option structs hold raw device addresses.  Each keeps a reference to the
+# tensors it points into (``_keep``), so that a struct built from a temporary dict does not
+# outlive its memory: a freed tensor's block is handed to the next allocation (a workspace,
+# say), and the library would then read that as weights.  A struct copied into another one
+# (``lw.router = ...``) or into a ctypes array does not carry the reference: the outer struct
+# or the caller's list does.
 def router_weights(w: dict) -> VpRouterWeights:
-    return VpRouterWeights(_p(w["r_W"]), _p(w["r_U"]), _p(w["r_w"]), _p(w.get("r_bW")),
-                           _p(w.get("r_bU")), _p(w.get("r_beta")))
+    rw = VpRouterWeights(_p(w["r_W"]), _p(w["r_U"]), _p(w["r_w"]), _p(w.get("r_bW")),
+                         _p(w.get("r_bU")), _p(w.get("r_beta")))
+    rw._keep = w
+    return rw
 
 
 def surrogate_weights(w: dict) -> VpSurrogateWeights:
-    return VpSurrogateWeights(*[_p(w[k]) for k in ("s_g1_w", "s_g1_b", "s_g2_w", "s_g2_b",
-                                                    "s_d1_w", "s_d1_b", "s_d2_w", "s_d2_b")])
+    sw = VpSurrogateWeights(*[_p(w[k]) for k in ("s_g1_w", "s_g1_b", "s_g2_w", "s_g2_b",
+                                                  "s_d1_w", "s_d1_b", "s_d2_w", "s_d2_b")])
+    sw._keep = w
+    return sw
 
 
 def qk_options(w: dict = None, norm_eps: float = 1e-6, rope: bool = False, tokens_per_view: int = 1,
@@ -166,12 +176,15 @@ def qk_options(w: dict = None, norm_eps: float = 1e-6, rope: bool = False, token
     o.patch_start = patch_start
     o.grid_w = grid_w
     o.rope_base = rope_base
+    o._keep = w
     return o
 
 
 def merge_options(stride: int, tokens_per_view: int, patch_start: int = 5, assign_out=None) -> VpMergeOptions:
     """vp_merge_options; assign_out: int32 device tensor [N] or None."""
-    return VpMergeOptions(stride, tokens_per_view, patch_start, _p(assign_out))
+    mo = VpMergeOptions(stride, tokens_per_view, patch_start, _p(assign_out))
+    mo._keep = assign_out
+    return mo
 
 
 def layer_weights(w: dict, qk: VpQkOptions = None, merge: VpMergeOptions = None) -> VpLayerWeights:
@@ -180,6 +193,7 @@ def layer_weights(w: dict, qk: VpQkOptions = None, merge: VpMergeOptions = None)
                                              "ls2")])
     lw.router = router_weights(w)
     lw.surrogate = surrogate_weights(w)
+    lw._keep = w
     if qk is not None:
         lw.qk = ctypes.pointer(qk)
         lw._qk_keep = qk  # the struct must outlive the call

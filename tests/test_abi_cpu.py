@@ -166,3 +166,46 @@ def test_option_struct_layouts(vp):
     assert ctypes.sizeof(vp.VpQkOptions) == 4 * 8 + 4 + 4 * 4 + 4
     assert ctypes.sizeof(vp.VpMergeOptions) == 3 * 4 + 4 + 8
     assert ctypes.sizeof(vp.VpLayerWeights) == 14 * 8 + 6 * 8 + 8 * 8 + 2 * 8
+
+
+def test_weight_structs_keep_their_tensors(vp):
+    """A struct built from a temporary dict keeps the buffers it points into alive: freed,
+    their memory would go to the next allocation and be read as weights.  (Stand-in buffers
+    that only carry an address: the binding takes device tensors, and there is no device here.)"""
+    import gc
+    import weakref
+
+    import synth
+
+    class Buf:  # an address, like a device tensor's data_ptr()
+        def __init__(self, addr):
+            self.addr = addr
+
+        def __int__(self):
+            return self.addr
+
+    names = list(synth.make_layer_weights(synth.rng(3), block=True)) + ["q_norm_g", "q_norm_b"]
+
+    def fresh():
+        return {k: Buf(4096 * (i + 1)) for i, k in enumerate(names)}
+
+    built, refs = {}, {}
+    for kind, make in (("layer", vp.layer_weights), ("router", vp.router_weights),
+                       ("surrogate", vp.surrogate_weights), ("qk", vp.qk_options)):
+        w = fresh()
+        refs[kind] = weakref.ref(w["r_U"] if kind == "router" else w["s_d2_b"] if kind == "surrogate"
+                                 else w["q_norm_g"] if kind == "qk" else w["b_qkv"])
+        built[kind] = make(w)
+        del w
+    assign = Buf(1 << 30)
+    refs["merge"] = weakref.ref(assign)
+    built["merge"] = vp.merge_options(4, 261, 5, assign)
+    del assign
+    gc.collect()
+    for kind, r in refs.items():
+        assert r() is not None, kind
+    assert built["layer"].b_qkv == int(refs["layer"]())
+    assert built["router"].U == int(refs["router"]())
+    assert built["surrogate"].d2_b == int(refs["surrogate"]())
+    assert built["qk"].q_norm_g == int(refs["qk"]())
+    assert built["merge"].assign_out == 1 << 30

@@ -127,7 +127,8 @@ def test_single_view_merges_nothing():
     force = np.array([[2, 1, 0, 1] * 4])
     dm = vpb.dims(N, 16)
     assign = torch.full((N,), -1, dtype=torch.int32, device="cuda")
-    layers = [vpb.layer_weights(vpb.to_device(w), None, vpb.merge_options(4, P224, 5, assign))]
+    dw = vpb.to_device(w)
+    layers = [vpb.layer_weights(dw, None, vpb.merge_options(4, P224, 5, assign))]
     ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
     x = vpb.bf16_from_bits(x_bits)
     modes = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
