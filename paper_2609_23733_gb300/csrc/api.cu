@@ -176,7 +176,8 @@ size_t stack_ws_bytes(const vp_dims* dm) {
 // membership tables, the merged tokens and their attention output.
 size_t merge_scratch_bytes(size_t N, size_t D) {
   return align_up(64 * D * 2) + align_up(64 * sizeof(float)) + 3 * align_up(N * 64 * 2) +
-         7 * align_up((N + 1) * sizeof(int)) + 2 * align_up(N * D * 2);
+         7 * align_up((N + 1) * sizeof(int)) + align_up(N * sizeof(unsigned long long)) +
+         2 * align_up(N * D * 2);
 }
 
 size_t stack_merge_ws_bytes(const vp_dims* dm) {
@@ -665,7 +666,7 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     p += align_up(64 * D * 2);
     ms.bbar = reinterpret_cast<float*>(p);
     p += align_up(64 * sizeof(float));
-    __nv_bfloat16** rows64[3] = {&ms.kbar, &ms.m, &ms.m_dst};
+    __nv_bfloat16** rows64[3] = {&ms.kbar, &ms.m_src, &ms.m_dst};
     for (__nv_bfloat16** q : rows64) {
       *q = reinterpret_cast<__nv_bfloat16*>(p);
       p += align_up(N * 64 * 2);
@@ -675,6 +676,8 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
       *q = reinterpret_cast<int*>(p);
       p += align_up((N + 1) * sizeof(int));
     }
+    ms.best = reinterpret_cast<unsigned long long*>(p);
+    p += align_up(N * sizeof(unsigned long long));
     ms.xm = reinterpret_cast<__nv_bfloat16*>(p);
     p += align_up(N * D * 2);
     ms.err = sc.err;

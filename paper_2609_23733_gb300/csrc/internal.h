@@ -167,15 +167,17 @@ cudaError_t launch_ln_fold_weights(int Nout, int K, const __nv_bfloat16* W, cons
 struct MergeGeo {
   int N, P, ps, stride;
   int Dv;  // destinations per view after the first
+  int Sv;  // sources per view after the first (P - Dv)
   int Np;  // merged tokens
+  int Ns;  // sources (N - Np)
 };
 MergeGeo make_merge_geo(int N, int P, int ps, int stride);
 struct MergeScratch {
   __nv_bfloat16* wbar;   // [64][D] head-mean key weights
   float* bbar;           // [64]
   __nv_bfloat16* kbar;   // [N][64] metric
-  __nv_bfloat16* m;      // [N][64] unit metric
-  __nv_bfloat16* m_dst;  // [Np][64]
+  __nv_bfloat16* m_src;  // [Ns][64] unit metric of the sources (in token order)
+  __nv_bfloat16* m_dst;  // [Np][64] unit metric of the destinations (by merged row)
   int* row_of;           // [N] merged row of a destination, -1 for sources
   int* dst_tok;          // [Np] token of merged row
   int* assign;           // [N] merged row every token joins
@@ -183,6 +185,7 @@ struct MergeScratch {
   int* offs;             // [Np + 1]
   int* fill;             // [Np]
   int* members;          // [N]
+  unsigned long long* best;  // [Ns] matching: (score, destination) keys, 0 before the matching
   __nv_bfloat16* xm;     // [Np][D] merged tokens
   unsigned int* err;
 };

@@ -9,10 +9,12 @@
 //     lowest destination), over all destinations of all views;
 //   merge: a merged token is the mean of its destination and the sources that joined it;
 //   unmerge: every token takes its merged token's attention output.
-// Kernels: the head-mean key weights, the metric GEMM (gemm_kernel), unit metric rows and the
-// destination table, the matching (tcgen05 scores of 128 sources x 256 destinations per MMA
-// group with a running argmax in the epilogue), counting / scan / fill of each merged token's members, their mean, and
-// the unmerge fused with LayerScale and the residual add.
+// Kernels: the head-mean key weights, the metric GEMM (gemm_kernel), unit metric rows of the
+// sources and of the destinations with the destination table, the matching (tcgen05 scores of
+// 128 sources x 256 destinations per MMA group with a running argmax in the epilogue, work
+// split evenly over the SMs), resolving and counting each token's merged row, scan and fill
+// of each merged token's members, their mean, and the unmerge fused with LayerScale and the
+// residual add.
 #include <math.h>
 
 #include "common.cuh"
@@ -33,6 +35,13 @@ __device__ __forceinline__ int merged_row(const MergeGeo& g, int i) {
   return p % g.stride == 0 ? base + g.ps + p / g.stride : -1;
 }
 
+// Sources in token order: view v >= 1 holds Sv = P - Dv of them, the patches q = t - ps with
+// q % stride != 0.  Index of source token i (merged_row(g, i) < 0) among all sources:
+__device__ __forceinline__ int source_index(const MergeGeo& g, int i) {
+  const int v = i / g.P, q = i - v * g.P - g.ps;
+  return (v - 1) * g.Sv + q - q / g.stride - 1;
+}
+
 // Head-mean key weights: wbar[c][k] = mean_h W_qkv[D + 64 h + c][k], bbar[c] likewise.
 __global__ void metric_weights_kernel(const __nv_bfloat16* w_qkv, const float* b_qkv, int H,
                                       int D, __nv_bfloat16* wbar, float* bbar) {
@@ -50,9 +59,10 @@ __global__ void metric_weights_kernel(const __nv_bfloat16* w_qkv, const float* b
   }
 }
 
-// One warp per token: the metric row as a unit vector (bf16), the merged row of every token
-// (-1 for sources), and for destinations their metric row and token index by merged row.
-__global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_bfloat16* m,
+// One warp per token: the metric row as a unit vector (bf16), stored by source index for a
+// source and by merged row for a destination; the merged row of every token (-1 for sources)
+// and the token of every merged row.
+__global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_bfloat16* m_src,
                                    __nv_bfloat16* m_dst, int* row_of, int* dst_tok) {
   const int lane = threadIdx.x & 31;
   const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -64,75 +74,98 @@ __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_b
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   const float inv = ss > 0.f ? rsqrtf(ss) : 0.f;
   const uint32_t mu = pack_bf16x2(a * inv, b * inv);
-  reinterpret_cast<uint32_t*>(m + (size_t)i * 64)[lane] = mu;
   const int r = merged_row(g, i);
-  if (r >= 0) reinterpret_cast<uint32_t*>(m_dst + (size_t)r * 64)[lane] = mu;
+  __nv_bfloat16* dst = r >= 0 ? m_dst + (size_t)r * 64 : m_src + (size_t)source_index(g, i) * 64;
+  reinterpret_cast<uint32_t*>(dst)[lane] = mu;
   if (lane == 0) {
     row_of[i] = r;
     if (r >= 0) dst_tok[r] = i;
   }
 }
 
-// Matching on the tensor cores: scores S = M_src M_dst^T (cosines of unit keys) for 128 source
-// rows at a time against chunks of 256 destinations, with a running argmax over the chunks.
-// Persistent CTAs (one per SM) take source tiles t = blockIdx.x, + gridDim.x, ...
-//   warp 0      TMA: the tile's 128 source rows once (16 KB), destination chunks (256 rows x
-//               64 channels, 32 KB, 128-byte swizzle) through a kMatchStages ring;
+// Matching on the tensor cores: scores S = M_src M_dst^T (cosines of unit keys) of 128 source
+// rows against chunks of 256 destinations, with a running argmax over the chunks.  The work
+// units (source tile, destination chunk) are split evenly over the CTAs (one per SM): CTA b
+// takes units [b U / G, (b + 1) U / G), runs of ascending chunks of one tile or more
+// (segments), so that no SM idles through a partial last round.  Each segment's best per row
+// goes into a 64-bit atomic maximum of (score, lowest column), which also joins the rows whose
+// chunks two CTAs share.
+//   warp 0      TMA: a segment's 128 source rows (16 KB, two buffers) and destination chunks
+//               (256 rows x 64 channels, 32 KB, 128-byte swizzle) through a kMatchStages ring;
 //   warp 1      TMEM owner and MMA issue: four tcgen05.mma M128 N256 K16 per chunk into one
 //               of two 256-column fp32 accumulators (the epilogue of one chunk overlaps the
 //               MMAs of the next);
 //   warps 4-19  argmax: a source row (TMEM lane) and a quarter of each chunk's columns per
-//               thread, 32 columns per tcgen05.ld (the next in flight), the max of the 32 by
-//               a tree first and the column only when it reaches the row's best (equal
-//               scores go to the lower index); the four parts combine at the end of the tile.
+//               thread, 32 columns (a piece) per tcgen05.ld, the next in flight.  A tree gives
+//               the piece's max; a piece whose max beats the row's best is copied to the
+//               thread's slot in shared memory, and the column is looked up there once, at the
+//               end of the segment.  Chunks ascend within a segment, so the first piece that
+//               reaches a score holds its lowest column.
 constexpr int kMatchStages = 4;
 constexpr int kMatchN = 256;
-constexpr int kMatchParts = 4;  // column parts of a chunk (argmax warps per TMEM lane quarter)
-constexpr int kMatchThreads = 128 + 128 * kMatchParts;
+constexpr int kMatchParts = 4;                // column parts of a chunk (argmax warps per TMEM lane quarter)
+constexpr int kMatchWarps = 4 * kMatchParts;  // argmax warps
+constexpr int kMatchThreads = 128 + 32 * kMatchWarps;
 constexpr uint32_t kMatchTmemCols = 512;
 
 struct MatchSmem {
-  __nv_bfloat16 src[128 * 64];
+  __nv_bfloat16 src[2][128 * 64];
   __nv_bfloat16 dst[kMatchStages][kMatchN * 64];
-  uint64_t src_full, src_empty;
+  float4 stash[kMatchWarps][32][8];  // each argmax thread's best piece, 16-byte slots rotated by lane
+  uint64_t src_full[2], src_empty[2];
   uint64_t dst_full[kMatchStages], dst_empty[kMatchStages];
   uint64_t acc_full[2], acc_empty[2], drain;
-  uint64_t part_post, part_taken;  // parts 1.. posted their best / part 0 read them
-  float part_v[kMatchParts - 1][128];  // parts 1..'s best per row, for the combine
-  int part_i[kMatchParts - 1][128];
   uint32_t tmem_base;
   int abort_flag;
 };
 
+// The run of units starting at unit u of a CTA's range [u, u_end): tile t, chunks [c0, c1).
+struct Segment {
+  int t, c0, c1;
+};
+__device__ __forceinline__ Segment segment_at(long long u, long long u_end, int n_chunks) {
+  Segment sg;
+  sg.t = (int)(u / n_chunks);
+  sg.c0 = (int)(u - (long long)sg.t * n_chunks);
+  sg.c1 = (int)min((long long)n_chunks, (long long)sg.c0 + (u_end - u));
+  return sg;
+}
+
+// (score, column) as one 64-bit key that orders like the argmax: higher score first, then the
+// lower column.  Float bits made monotone: negative values inverted, positive ones offset.
+__device__ __forceinline__ unsigned long long match_key(float v, int col) {
+  const uint32_t b = __float_as_uint(v);
+  const uint32_t ord = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+  return ((unsigned long long)ord << 32) | (unsigned long long)(~(uint32_t)col);
+}
+
 __global__ void __launch_bounds__(kMatchThreads, 1)
     tome_match_kernel(const __grid_constant__ CUtensorMap tmap_src,
-                      const __grid_constant__ CUtensorMap tmap_dst, MergeGeo g, const int* row_of,
-                      int* assign, unsigned int* err) {
+                      const __grid_constant__ CUtensorMap tmap_dst, MergeGeo g,
+                      unsigned long long* best, unsigned int* err) {
   extern __shared__ unsigned char smem_raw[];
   MatchSmem& sm = *reinterpret_cast<MatchSmem*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  const int n_tiles = (g.N + 127) / 128;
+  const int n_tiles = (g.Ns + 127) / 128;
   const int n_chunks = (g.Np + kMatchN - 1) / kMatchN;
-  if ((int)blockIdx.x >= n_tiles) return;
-  // The CTAs sweep the destination chunks from staggered starts, so that they do not all
-  // read the same chunk (the same L2 lines) at the same time.
-  const int ch_start = (int)(((long long)blockIdx.x * n_chunks) / gridDim.x);
+  const long long n_units = (long long)n_tiles * n_chunks;
+  const long long u_begin = n_units * blockIdx.x / gridDim.x;
+  const long long u_end = n_units * (blockIdx.x + 1) / gridDim.x;
+  if (u_begin >= u_end) return;  // uniform across the CTA
   const int warp = warp_uniform_id(), lane = lane_id();
   volatile int* abort_flag = &sm.abort_flag;
   if (threadIdx.x == 0) {
-    mbar_init(&sm.src_full, 1);
-    mbar_init(&sm.src_empty, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.src_full[b], 1);
+      mbar_init(&sm.src_empty[b], 1);
+      mbar_init(&sm.acc_full[b], 1);
+      mbar_init(&sm.acc_empty[b], 32 * kMatchWarps);
+    }
     for (int s = 0; s < kMatchStages; ++s) {
       mbar_init(&sm.dst_full[s], 1);
       mbar_init(&sm.dst_empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&sm.acc_full[b], 1);
-      mbar_init(&sm.acc_empty[b], 128 * kMatchParts);
-    }
     mbar_init(&sm.drain, 1);
-    mbar_init(&sm.part_post, 128 * (kMatchParts - 1));
-    mbar_init(&sm.part_taken, 128);
     sm.abort_flag = 0;
     fence_mbarrier_init();
     fence_proxy_async_smem();
@@ -150,31 +183,38 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    uint32_t lc = 0, ic = 0;
+    uint32_t lc = 0, sc = 0;  // destination chunks / source tiles issued
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ic) {
-      ok = mbar_wait_warp(&sm.src_empty, (ic & 1) ^ 1, err, abort_flag);
+    for (long long u = u_begin; u < u_end && ok;) {
+      const Segment sg = segment_at(u, u_end, n_chunks);
+      const int sb = sc & 1;
+      ok = mbar_wait_warp(&sm.src_empty[sb], ((sc >> 1) & 1) ^ 1, err, abort_flag);
       if (!ok) break;
       if (elect_one()) {
-        mbar_arrive_expect_tx(&sm.src_full, 128 * 64 * 2);
-        tma_load_2d(sm.src, &tmap_src, &sm.src_full, 0, t * 128);
+        mbar_arrive_expect_tx(&sm.src_full[sb], 128 * 64 * 2);
+        tma_load_2d(sm.src[sb], &tmap_src, &sm.src_full[sb], 0, sg.t * 128);
       }
       __syncwarp();
-      for (int ch = 0; ch < n_chunks; ++ch, ++lc) {
+      ++sc;
+      for (int ch = sg.c0; ch < sg.c1; ++ch, ++lc) {
         const int st = lc % kMatchStages;
         ok = mbar_wait_warp(&sm.dst_empty[st], ((lc / kMatchStages) & 1) ^ 1, err, abort_flag);
         if (!ok) break;
         if (elect_one()) {
-          const int chunk = (ch_start + ch) % n_chunks;
           mbar_arrive_expect_tx(&sm.dst_full[st], kMatchN * 64 * 2);
-          tma_load_2d(sm.dst[st], &tmap_dst, &sm.dst_full[st], 0, chunk * kMatchN);
+          tma_load_2d(sm.dst[st], &tmap_dst, &sm.dst_full[st], 0, ch * kMatchN);
         }
         __syncwarp();
       }
+      u += sg.c1 - sg.c0;
     }
     if (!ok && lane == 0) {  // let issued copies land before the CTA releases its smem
-      if (ic > 0)
-        for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.src_full, (ic - 1) & 1); ++k) {}
+      for (int b = 0; b < 2; ++b) {
+        if (sc > (uint32_t)b) {
+          const uint32_t last = (sc - 1 - b) / 2 * 2 + b;  // last tile load into buffer b
+          for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.src_full[b], (last >> 1) & 1); ++k) {}
+        }
+      }
       for (int s = 0; s < kMatchStages; ++s) {
         if (lc > (uint32_t)s) {
           const uint32_t last = (lc - 1 - s) / kMatchStages * kMatchStages + s;
@@ -185,14 +225,16 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issue
     const uint32_t idesc = idesc_bf16(128, kMatchN, 0, 0);
-    const uint64_t da = sdesc_sw128(smem_u32(sm.src));
-    uint32_t lc = 0, ic = 0, ac = 0;
+    uint32_t lc = 0, sc = 0, ac = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ic) {
-      ok = mbar_wait_warp(&sm.src_full, ic & 1, err, abort_flag);
+    for (long long u = u_begin; u < u_end && ok; ++sc) {
+      const Segment sg = segment_at(u, u_end, n_chunks);
+      const int sb = sc & 1;
+      ok = mbar_wait_warp(&sm.src_full[sb], (sc >> 1) & 1, err, abort_flag);
       if (!ok) break;
       tc_fence_after();
-      for (int ch = 0; ch < n_chunks; ++ch, ++lc, ++ac) {
+      const uint64_t da = sdesc_sw128(smem_u32(sm.src[sb]));
+      for (int ch = sg.c0; ch < sg.c1; ++ch, ++lc, ++ac) {
         const int st = lc % kMatchStages;
         const uint32_t ab = ac & 1;
         ok = mbar_wait_warp(&sm.dst_full[st], (lc / kMatchStages) & 1, err, abort_flag) &&
@@ -206,10 +248,11 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
             tc_mma_ss(tmem + ab * kMatchN, da + 2 * kk, db + 2 * kk, idesc, kk > 0 ? 1u : 0u);
           tc_commit(&sm.acc_full[ab]);
           tc_commit(&sm.dst_empty[st]);
-          if (ch == n_chunks - 1) tc_commit(&sm.src_empty);
+          if (ch == sg.c1 - 1) tc_commit(&sm.src_empty[sb]);
         }
         __syncwarp();
       }
+      u += sg.c1 - sg.c0;
     }
     if (!ok) {
       if (elect_one()) {
@@ -221,21 +264,24 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
   } else if (warp >= 4) {
     // ------------------------------------------------------------ running argmax
     constexpr int kCols = kMatchN / kMatchParts;  // columns of a part
-    const int quarter = warp & 3, part = (warp - 4) >> 2;
+    const int aw = warp - 4;
+    const int quarter = warp & 3, part = aw >> 2;
     const int rit = quarter * 32 + lane;  // row in the tile
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16) + part * kCols;
-    uint32_t ac = 0, ic = 0;
+    float4* slot = sm.stash[aw][lane];
+    uint32_t ac = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ic) {
+    for (long long u = u_begin; u < u_end && ok;) {
+      const Segment sg = segment_at(u, u_end, n_chunks);
       float bv = -INFINITY;
-      int bi = 0x7fffffff;
-      for (int ch = 0; ch < n_chunks; ++ch, ++ac) {
+      int bcol = -1;  // first column of the stashed piece
+      for (int ch = sg.c0; ch < sg.c1; ++ch, ++ac) {
         const uint32_t ab = ac & 1;
         ok = mbar_wait_warp(&sm.acc_full[ab], (ac >> 1) & 1, err, abort_flag);
         if (!ok) break;
         tc_fence_after();
-        const int c0 = ((ch_start + ch) % n_chunks) * kMatchN + part * kCols;  // first destination
-        const int valid = g.Np - c0;                         // columns past it hold no destination
+        const int c0 = ch * kMatchN + part * kCols;  // first destination of the part
+        const int valid = g.Np - c0;                 // columns past it hold no destination
         float v[2][32];
         tmem_ld32(t_lane + ab * kMatchN, v[0]);
         tmem_wait_ld();
@@ -256,15 +302,12 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
 #pragma unroll
             for (int e = 0; e < 4; ++e) q[e] = fmax3(q[e], x[k + e], x[k + 4 + e]);
           const float mx = fmax3(q[0], q[1], fmaxf(q[2], q[3]));
-          if (mx >= bv) {  // chunks come in rotated order: equal scores go to the lower index
-            int best = 0;
+          if (mx > bv) {  // a strictly better piece: keep its scores
+            bv = mx;
+            bcol = c0 + 32 * p;
 #pragma unroll
-            for (int k = 31; k >= 0; --k)
-              if (x[k] == mx) best = c0 + 32 * p + k;
-            if (mx > bv || best < bi) {
-              bv = mx;
-              bi = best;
-            }
+            for (int j = 0; j < 8; ++j)
+              slot[(j + lane) & 7] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
           }
           tmem_wait_ld();
         }
@@ -272,31 +315,23 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
         mbar_arrive(&sm.acc_empty[ab]);
       }
       if (!ok) break;
-      // Combine the parts through shared memory and two mbarriers (bounded waits): parts 1..
-      // post their best once part 0 has read the previous tile's; part 0 decides (larger
-      // score, then lower index).
-      if (part > 0) {
-        ok = mbar_wait_warp(&sm.part_taken, (ic & 1) ^ 1, err, abort_flag);
-        if (!ok) break;
-        sm.part_v[part - 1][rit] = bv;
-        sm.part_i[part - 1][rit] = bi;
-        mbar_arrive(&sm.part_post);
-      } else {
-        ok = mbar_wait_warp(&sm.part_post, ic & 1, err, abort_flag);
-        if (!ok) break;
+      u += sg.c1 - sg.c0;
+      const int row = sg.t * 128 + rit;
+      if (bcol >= 0 && row < g.Ns) {  // the lowest column of the kept piece that holds bv
+        float x[32];
 #pragma unroll
-        for (int q = 0; q < kMatchParts - 1; ++q) {
-          const float ov = sm.part_v[q][rit];
-          const int oi = sm.part_i[q][rit];
-          if (ov > bv || (ov == bv && oi < bi)) {
-            bv = ov;
-            bi = oi;
-          }
+        for (int j = 0; j < 8; ++j) {
+          const float4 f = slot[(j + lane) & 7];
+          x[4 * j] = f.x;
+          x[4 * j + 1] = f.y;
+          x[4 * j + 2] = f.z;
+          x[4 * j + 3] = f.w;
         }
-        mbar_arrive(&sm.part_taken);
-        const int row = t * 128 + rit;
-        if (bi >= g.Np) bi = 0;  // no score compared (NaN metric): any valid row
-        if (row < g.N) assign[row] = row_of[row] >= 0 ? row_of[row] : bi;
+        int k_best = 31;
+#pragma unroll
+        for (int k = 31; k >= 0; --k)
+          if (x[k] == bv) k_best = k;
+        atomicMax(best + row, match_key(bv, bcol + k_best));
       }
     }
   }
@@ -308,34 +343,77 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
   }
 }
 
-__global__ void merge_count_kernel(int N, const int* assign, int* cnt) {
+// The merged row of every token -- its own for a destination, the matched destination for a
+// source -- counted per merged row.
+__global__ void merge_resolve_kernel(MergeGeo g, const int* row_of, const unsigned long long* best,
+                                     int* assign, int* cnt) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < N) atomicAdd(cnt + assign[i], 1);
+  if (i >= g.N) return;
+  int r = row_of[i];
+  if (r < 0) {
+    const unsigned long long k = best[source_index(g, i)];
+    r = k ? (int)~(uint32_t)k : 0;  // no score compared (NaN metric): any valid row
+    if (r < 0 || r >= g.Np) r = 0;
+  }
+  assign[i] = r;
+  atomicAdd(cnt + r, 1);
 }
 
-// Exclusive scan of cnt[0..n) into offs[0..n] in one block of 1024 threads: each thread sums
-// a contiguous run, the block scans the run totals, then each thread writes its run.
+// Exclusive scan of cnt[0..n) into offs[0..n] in one block of 1024 threads, 4,096 entries a
+// round: four per thread (one 16-byte load, the next round's in flight), a warp scan of the
+// thread totals, a scan of the 32 warp totals, and the carry of the rounds before.
 __global__ void __launch_bounds__(1024) scan_kernel(int n, const int* cnt, int* offs) {
-  __shared__ int part[1024];
-  const int tid = threadIdx.x;
-  const int per = (n + 1023) / 1024;
-  const int b = min(n, tid * per), e = min(n, b + per);
-  int s = 0;
-  for (int k = b; k < e; ++k) s += cnt[k];
-  part[tid] = s;
-  __syncthreads();
-  for (int o = 1; o < 1024; o <<= 1) {  // Hillis-Steele inclusive scan
-    const int v = tid >= o ? part[tid - o] : 0;
+  __shared__ int warp_ex[32];
+  __shared__ int round_total;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  auto load4 = [&](int base) {
+    const int i = base + 4 * tid;
+    if (i + 3 < n) return *reinterpret_cast<const int4*>(cnt + i);
+    int4 r = make_int4(0, 0, 0, 0);
+    if (i < n) r.x = cnt[i];
+    if (i + 1 < n) r.y = cnt[i + 1];
+    if (i + 2 < n) r.z = cnt[i + 2];
+    return r;
+  };
+  int carry = 0;
+  int4 nxt = load4(0);
+  for (int base = 0; base < n; base += 4096) {
+    const int4 c = nxt;
+    if (base + 4096 < n) nxt = load4(base + 4096);
+    const int s1 = c.x, s2 = s1 + c.y, s3 = s2 + c.z, tot = s3 + c.w;
+    int incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_ex[wid] = incl;
     __syncthreads();
-    part[tid] += v;
+    if (wid == 0) {
+      const int w = warp_ex[lane];
+      int wi = w;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, wi, o);
+        if (lane >= o) wi += y;
+      }
+      warp_ex[lane] = wi - w;
+      if (lane == 31) round_total = wi;
+    }
     __syncthreads();
+    const int ex = carry + warp_ex[wid] + incl - tot;
+    const int i = base + 4 * tid;
+    if (i + 3 < n) {
+      *reinterpret_cast<int4*>(offs + i) = make_int4(ex, ex + s1, ex + s2, ex + s3);
+    } else {
+      if (i < n) offs[i] = ex;
+      if (i + 1 < n) offs[i + 1] = ex + s1;
+      if (i + 2 < n) offs[i + 2] = ex + s2;
+    }
+    carry += round_total;
+    __syncthreads();  // warp_ex and round_total are rewritten in the next round
   }
-  int run = part[tid] - s;
-  for (int k = b; k < e; ++k) {
-    offs[k] = run;
-    run += cnt[k];
-  }
-  if (tid == 1023) offs[n] = part[1023];
+  if (tid == 0) offs[n] = carry;
 }
 
 __global__ void merge_fill_kernel(int N, const int* assign, const int* offs, int* fill,
@@ -438,7 +516,9 @@ MergeGeo make_merge_geo(int N, int P, int ps, int stride) {
   g.ps = ps;
   g.stride = stride;
   g.Dv = ps + (P - ps + stride - 1) / stride;
+  g.Sv = P - g.Dv;
   g.Np = N <= P ? N : P + (N / P - 1) * g.Dv;
+  g.Ns = N - g.Np;
   return g;
 }
 
@@ -464,28 +544,37 @@ cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* 
   e = launch_linear(la, num_sms, st);
   if (e != cudaSuccess) return e;
   prof_before(VP_KERNEL_MERGE, st);
-  merge_setup_kernel<<<(g.N + 7) / 8, 256, 0, st>>>(g, s.kbar, s.m, s.m_dst, s.row_of, s.dst_tok);
+  merge_setup_kernel<<<(g.N + 7) / 8, 256, 0, st>>>(g, s.kbar, s.m_src, s.m_dst, s.row_of,
+                                                     s.dst_tok);
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  CUtensorMap tsrc, tdst;  // unit metric rows, 64 channels (128 bytes), 128-byte swizzle
-  if ((e = make_tmap_bf16_2d(&tsrc, s.m, 64, (uint64_t)g.N, 64, 64, 128)) != cudaSuccess) return e;
-  if ((e = make_tmap_bf16_2d(&tdst, s.m_dst, 64, (uint64_t)g.Np, 64, 64, kMatchN)) != cudaSuccess)
-    return e;
-  const int smem = (int)sizeof(MatchSmem) + 1024;
-  if ((e = cudaFuncSetAttribute(tome_match_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                smem)) != cudaSuccess)
-    return e;
-  prof_before(VP_KERNEL_MERGE, st);
-  tome_match_kernel<<<min(num_sms, (g.N + 127) / 128), kMatchThreads, smem, st>>>(
-      tsrc, tdst, g, s.row_of, s.assign, s.err);
-  prof_after(st);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  if (g.Ns > 0) {  // one view, or stride 1: every token is a destination
+    CUtensorMap tsrc, tdst;  // unit metric rows, 64 channels (128 bytes), 128-byte swizzle
+    if ((e = make_tmap_bf16_2d(&tsrc, s.m_src, 64, (uint64_t)g.Ns, 64, 64, 128)) != cudaSuccess)
+      return e;
+    if ((e = make_tmap_bf16_2d(&tdst, s.m_dst, 64, (uint64_t)g.Np, 64, 64, kMatchN)) != cudaSuccess)
+      return e;
+    const int smem = (int)sizeof(MatchSmem) + 1024;
+    if ((e = cudaFuncSetAttribute(tome_match_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem)) != cudaSuccess)
+      return e;
+    const long long units =
+        (long long)((g.Ns + 127) / 128) * ((g.Np + kMatchN - 1) / kMatchN);
+    prof_before(VP_KERNEL_MERGE, st);
+    e = cudaMemsetAsync(s.best, 0, (size_t)g.Ns * sizeof(unsigned long long), st);
+    if (e == cudaSuccess) {
+      tome_match_kernel<<<(int)min((long long)num_sms, units), kMatchThreads, smem, st>>>(
+          tsrc, tdst, g, s.best, s.err);
+      e = cudaGetLastError();
+    }
+    prof_after(st);
+    if (e != cudaSuccess) return e;
+  }
   if ((e = cudaMemsetAsync(s.cnt, 0, (size_t)g.Np * sizeof(int), st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(s.fill, 0, (size_t)g.Np * sizeof(int), st)) != cudaSuccess) return e;
   prof_before(VP_KERNEL_MERGE, st);
-  merge_count_kernel<<<(g.N + 255) / 256, 256, 0, st>>>(g.N, s.assign, s.cnt);
+  merge_resolve_kernel<<<(g.N + 255) / 256, 256, 0, st>>>(g, s.row_of, s.best, s.assign, s.cnt);
   scan_kernel<<<1, 1024, 0, st>>>(g.Np, s.cnt, s.offs);
   merge_fill_kernel<<<(g.N + 255) / 256, 256, 0, st>>>(g.N, s.assign, s.offs, s.fill, s.members);
   prof_extra_launch();
