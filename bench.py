@@ -623,14 +623,14 @@ def kernel_case(args):
         z = torch.zeros(H, d, device=dev)
         for _ in range(args.case_launches):
             vpb.vp_head_attention(dm, qkv, ids, off, z, z, vpb.surrogate_weights(w), y, ws)
-    elif args.kernel_case == "merge":  # one block with token merging (stride 10) over whole views
+    elif args.kernel_case == "merge":  # one block with token merging over whole views
         P = synth.tokens_per_view(518)
         Nm = max(1, N // P) * P
         w = vpb.to_device(synth.make_layer_weights(synth.rng(0), block=True), dev)
         dm = vpb.dims(Nm, H)
         ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE, dev)
         x = torch.randn(Nm, D, device=dev).to(torch.bfloat16)
-        layer = [vpb.layer_weights(w, None, vpb.merge_options(10, P, 5))]
+        layer = [vpb.layer_weights(w, None, vpb.merge_options(args.case_stride, P, 5))]
         fm = torch.tensor([synth.forced_mix(H, 0.25)], dtype=torch.int32, device=dev)
         modes = torch.zeros(1, H, dtype=torch.int32, device=dev)
         s = torch.zeros(1, H, device=dev)
@@ -700,6 +700,7 @@ def main():
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
     ap.add_argument("--case-tokens", type=int, default=32768)
     ap.add_argument("--case-launches", type=int, default=2)
+    ap.add_argument("--case-stride", type=int, default=10, help="token-merging stride of --kernel-case merge")
     args = ap.parse_args()
     if args.kernel_case:
         kernel_case(args)

@@ -722,7 +722,9 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
       const QkArgs qm{w.qk, rope, ms.dst_tok};
       VP_TRY(run_layer(&dm, ms.xm, w.w_qkv, w.b_qkv, w.w_o, w.b_o, nullptr, nullptr, &w.router,
                        &w.surrogate, fm, merged_out, qkv, y, s_l, sa_l, m_l, sc, st, nullptr, &qm));
-      VP_TRY(from_cuda(launch_unmerge_residual(dims->N, D, ms.assign, merged_out, w.ls1, x, st)));
+      // unmerge, X_attn = X + LS1 (.) A, and (4)'s Z~ = LN2(X_attn) in one pass
+      VP_TRY(from_cuda(launch_unmerge_ln(dims->N, D, ms.assign, merged_out, w.ls1, w.ln2_g,
+                                         w.ln2_b, ln_eps, x, zt, st)));
     } else {
       const QkArgs qa{w.qk, rope, nullptr};
       // (1)-(3) X <- X + LS1 (Y W_O + b_O) in place, Y the routed attention of LN1(X)
@@ -730,8 +732,9 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
       VP_TRY(run_layer(dims, x, reinterpret_cast<const vp_bf16*>(wq), bq, w.w_o, w.b_o, w.ls1, x,
                        &w.router, &w.surrogate, fm, x, qkv, y, s_l, sa_l, m_l, sc, st, &fold, &qa));
     }
-    // (4) Z~ = LN2(X_attn); X <- X_attn + LS2 FFN(Z~)
-    VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, zt, st)));
+    // (4) Z~ = LN2(X_attn) (done above for a merged block); X <- X_attn + LS2 FFN(Z~)
+    if (!w.merge)
+      VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln2_g, w.ln2_b, ln_eps, zt, st)));
     LinearArgs f1{};
     f1.M = dims->N;
     f1.N = 4 * D;

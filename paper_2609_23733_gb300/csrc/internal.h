@@ -193,9 +193,11 @@ struct MergeScratch {
 cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* xt,
                                  const __nv_bfloat16* w_qkv, const float* b_qkv,
                                  const MergeScratch& s, int num_sms, cudaStream_t st);
-// x[i] += ls (.) a[assign[i]] over N rows of D channels.
-cudaError_t launch_unmerge_residual(int N, int D, const int* assign, const __nv_bfloat16* a,
-                                    const float* ls, __nv_bfloat16* x, cudaStream_t st);
+// x[i] = bf16(x[i] + ls (.) a[assign[i]]) and z[i] = LN(x[i]) (g, b, eps) over N rows of D
+// channels.
+cudaError_t launch_unmerge_ln(int N, int D, const int* assign, const __nv_bfloat16* a,
+                              const float* ls, const float* g, const float* b, float eps,
+                              __nv_bfloat16* x, __nv_bfloat16* z, cudaStream_t st);
 
 cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float* g,
                               const float* b, float eps, __nv_bfloat16* out, cudaStream_t st);

@@ -13,8 +13,8 @@
 // sources and of the destinations with the destination table, the matching (tcgen05 scores of
 // 128 sources x 256 destinations per MMA group with a running argmax in the epilogue, work
 // split evenly over the SMs), resolving and counting each token's merged row, scan and fill
-// of each merged token's members, their mean, and the unmerge fused with LayerScale and the
-// residual add.
+// of each merged token's members, their mean, and the unmerge fused with LayerScale, the
+// residual add and the block's second LayerNorm.
 #include <math.h>
 
 #include "common.cuh"
@@ -59,25 +59,32 @@ __global__ void metric_weights_kernel(const __nv_bfloat16* w_qkv, const float* b
   }
 }
 
-// One warp per token: the metric row as a unit vector (bf16), stored by source index for a
-// source and by merged row for a destination; the merged row of every token (-1 for sources)
-// and the token of every merged row.
+// Eight lanes per token (16 bytes each, four tokens per warp): the metric row as a unit vector
+// (bf16), stored by source index for a source and by merged row for a destination; the
+// merged row of every token (-1 for sources) and the token of every merged row.
 __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_bfloat16* m_src,
                                    __nv_bfloat16* m_dst, int* row_of, int* dst_tok) {
-  const int lane = threadIdx.x & 31;
-  const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (i >= g.N) return;
-  const uint32_t u = reinterpret_cast<const uint32_t*>(kbar + (size_t)i * 64)[lane];
-  const float a = bf16_lo(u), b = bf16_hi(u);
-  float ss = a * a + b * b;
+  const int sub = threadIdx.x & 7;
+  const int i = blockIdx.x * (blockDim.x >> 3) + (threadIdx.x >> 3);
+  if (i >= g.N) return;  // whole groups of eight lanes leave together
+  const uint4 u = reinterpret_cast<const uint4*>(kbar + (size_t)i * 64)[sub];
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  float ss = 0.f;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  for (int k = 0; k < 4; ++k) ss += bf16_lo(w[k]) * bf16_lo(w[k]) + bf16_hi(w[k]) * bf16_hi(w[k]);
+  // the warp's tokens that exist: a prefix of its four groups of eight lanes
+  const int live = min(4, g.N - (i - (int)((threadIdx.x & 31) >> 3)));
+  const unsigned mask = live == 4 ? 0xffffffffu : (1u << (8 * live)) - 1u;
+#pragma unroll
+  for (int o = 4; o > 0; o >>= 1) ss += __shfl_xor_sync(mask, ss, o);
   const float inv = ss > 0.f ? rsqrtf(ss) : 0.f;
-  const uint32_t mu = pack_bf16x2(a * inv, b * inv);
+  uint32_t mu[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) mu[k] = pack_bf16x2(bf16_lo(w[k]) * inv, bf16_hi(w[k]) * inv);
   const int r = merged_row(g, i);
   __nv_bfloat16* dst = r >= 0 ? m_dst + (size_t)r * 64 : m_src + (size_t)source_index(g, i) * 64;
-  reinterpret_cast<uint32_t*>(dst)[lane] = mu;
-  if (lane == 0) {
+  reinterpret_cast<uint4*>(dst)[sub] = make_uint4(mu[0], mu[1], mu[2], mu[3]);
+  if (sub == 0) {
     row_of[i] = r;
     if (r >= 0) dst_tok[r] = i;
   }
@@ -478,32 +485,78 @@ __global__ void __launch_bounds__(256, C <= 4 ? 3 : 1) merge_mean_kernel(int Np,
   }
 }
 
-// x[i] <- x[i] + ls (.) a[assign[i]]: the unmerge, LayerScale and residual add of the block's
-// attention branch; one warp per token.
+// The end of a merged block's attention branch and its second LayerNorm, one warp per token:
+// x[i] <- bf16(x[i] + ls (.) a[assign[i]]) (unmerge, LayerScale, residual add) and
+// z[i] = LN(x[i]) (gamma, beta, eps) from the stored bf16 values, in one pass over the rows
+// (the LayerNorm kernel's arithmetic: fp32 mean, then the biased variance about it).
 template <int C>
-__global__ void unmerge_residual_kernel(int N, const int* assign, const __nv_bfloat16* a,
-                                        const float* ls, __nv_bfloat16* x) {
+__global__ void __launch_bounds__(256, 4) unmerge_ln_kernel(int N, const int* assign,
+                                                            const __nv_bfloat16* a, const float* ls,
+                                                            const float* g, const float* b,
+                                                            float eps, __nv_bfloat16* x,
+                                                            __nv_bfloat16* z) {
   constexpr int D = 256 * C;
   const int lane = threadIdx.x & 31;
   const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (i >= N) return;
   const int r = assign[i];
+  uint4 ua[C], ux[C];
 #pragma unroll
   for (int c = 0; c < C; ++c) {
     const int col = (c * 32 + lane) * 8;
-    const uint4 ua = __ldg(reinterpret_cast<const uint4*>(a + (size_t)r * D + col));
-    uint4* px = reinterpret_cast<uint4*>(x + (size_t)i * D + col);
-    const uint4 ux = *px;
+    ua[c] = __ldg(reinterpret_cast<const uint4*>(a + (size_t)r * D + col));
+    ux[c] = *reinterpret_cast<const uint4*>(x + (size_t)i * D + col);
+  }
+  uint32_t o[4 * C];  // the new residual row, bf16 pairs
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const int col = (c * 32 + lane) * 8;
     const float4 l0 = __ldg(reinterpret_cast<const float4*>(ls + col));
     const float4 l1 = __ldg(reinterpret_cast<const float4*>(ls + col) + 1);
     const float lw[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
-    const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w}, wx[4] = {ux.x, ux.y, ux.z, ux.w};
-    uint32_t o[4];
+    const uint32_t wa[4] = {ua[c].x, ua[c].y, ua[c].z, ua[c].w};
+    const uint32_t wx[4] = {ux[c].x, ux[c].y, ux[c].z, ux[c].w};
 #pragma unroll
     for (int k = 0; k < 4; ++k)
-      o[k] = pack_bf16x2(fmaf(lw[2 * k], bf16_lo(wa[k]), bf16_lo(wx[k])),
-                         fmaf(lw[2 * k + 1], bf16_hi(wa[k]), bf16_hi(wx[k])));
-    *px = make_uint4(o[0], o[1], o[2], o[3]);
+      o[4 * c + k] = pack_bf16x2(fmaf(lw[2 * k], bf16_lo(wa[k]), bf16_lo(wx[k])),
+                                 fmaf(lw[2 * k + 1], bf16_hi(wa[k]), bf16_hi(wx[k])));
+    *reinterpret_cast<uint4*>(x + (size_t)i * D + col) =
+        make_uint4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4 * C; ++k) {
+    s += bf16_lo(o[k]);
+    s += bf16_hi(o[k]);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  const float mean = s * (1.f / D);
+  float q = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4 * C; ++k) {
+    const float t0 = bf16_lo(o[k]) - mean, t1 = bf16_hi(o[k]) - mean;
+    q += t0 * t0;
+    q += t1 * t1;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
+  const float rstd = rsqrtf(q * (1.f / D) + eps);
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const int col = (c * 32 + lane) * 8;
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(g + col));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(g + col) + 1);
+    const float4 b0 = __ldg(reinterpret_cast<const float4*>(b + col));
+    const float4 b1 = __ldg(reinterpret_cast<const float4*>(b + col) + 1);
+    const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+    uint32_t y[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      y[k] = pack_bf16x2((bf16_lo(o[4 * c + k]) - mean) * rstd * gg[2 * k] + bb[2 * k],
+                         (bf16_hi(o[4 * c + k]) - mean) * rstd * gg[2 * k + 1] + bb[2 * k + 1]);
+    *reinterpret_cast<uint4*>(z + (size_t)i * D + col) = make_uint4(y[0], y[1], y[2], y[3]);
   }
 }
 
@@ -544,8 +597,8 @@ cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* 
   e = launch_linear(la, num_sms, st);
   if (e != cudaSuccess) return e;
   prof_before(VP_KERNEL_MERGE, st);
-  merge_setup_kernel<<<(g.N + 7) / 8, 256, 0, st>>>(g, s.kbar, s.m_src, s.m_dst, s.row_of,
-                                                     s.dst_tok);
+  merge_setup_kernel<<<(g.N + 31) / 32, 256, 0, st>>>(g, s.kbar, s.m_src, s.m_dst, s.row_of,
+                                                      s.dst_tok);
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -595,15 +648,17 @@ cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* 
   return cudaGetLastError();
 }
 
-cudaError_t launch_unmerge_residual(int N, int D, const int* assign, const __nv_bfloat16* a,
-                                    const float* ls, __nv_bfloat16* x, cudaStream_t st) {
+cudaError_t launch_unmerge_ln(int N, int D, const int* assign, const __nv_bfloat16* a,
+                              const float* ls, const float* g, const float* b, float eps,
+                              __nv_bfloat16* x, __nv_bfloat16* z, cudaStream_t st) {
   prof_before(VP_KERNEL_MERGE, st);
+  const int grid = (N + 7) / 8;
   switch (D / 256) {
-    case 1: unmerge_residual_kernel<1><<<(N + 7) / 8, 256, 0, st>>>(N, assign, a, ls, x); break;
-    case 2: unmerge_residual_kernel<2><<<(N + 7) / 8, 256, 0, st>>>(N, assign, a, ls, x); break;
-    case 3: unmerge_residual_kernel<3><<<(N + 7) / 8, 256, 0, st>>>(N, assign, a, ls, x); break;
-    case 4: unmerge_residual_kernel<4><<<(N + 7) / 8, 256, 0, st>>>(N, assign, a, ls, x); break;
-    case 8: unmerge_residual_kernel<8><<<(N + 7) / 8, 256, 0, st>>>(N, assign, a, ls, x); break;
+    case 1: unmerge_ln_kernel<1><<<grid, 256, 0, st>>>(N, assign, a, ls, g, b, eps, x, z); break;
+    case 2: unmerge_ln_kernel<2><<<grid, 256, 0, st>>>(N, assign, a, ls, g, b, eps, x, z); break;
+    case 3: unmerge_ln_kernel<3><<<grid, 256, 0, st>>>(N, assign, a, ls, g, b, eps, x, z); break;
+    case 4: unmerge_ln_kernel<4><<<grid, 256, 0, st>>>(N, assign, a, ls, g, b, eps, x, z); break;
+    case 8: unmerge_ln_kernel<8><<<grid, 256, 0, st>>>(N, assign, a, ls, g, b, eps, x, z); break;
     default: prof_after(st); return cudaErrorInvalidValue;
   }
   prof_after(st);

@@ -140,3 +140,50 @@ def test_single_view_merges_nothing():
     want, _ = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w)], force_modes=force,
                                   merge=[{"stride": 4, "tokens_per_view": P224, "patch_start": 5}])
     compare(_f64(x), want, rel=BF16_STEP, what="single view with merging on")
+
+
+def test_matching_ties_go_to_the_lowest_destination():
+    """View 2 repeats view 0 token for token, so every destination of view 2 has a twin in
+    view 0 with the same metric row: a source whose best destination is such a pair has an
+    exact tie, which goes to the lower merged row (the view-0 twin).  The twins sit in
+    different 256-destination chunks, which the matching hands to different CTAs, so the tie
+    is settled by the (score, lowest row) atomic maximum across CTAs."""
+    N = 4 * P224
+    g = synth.rng(24)
+    w = synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1)
+    x_bits = synth.make_tokens(24, N)
+    x_bits[2 * P224:3 * P224] = x_bits[:P224]
+    dm = vpb.dims(N, 16)
+    assign = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    dw = vpb.to_device(w)
+    layers = [vpb.layer_weights(dw, None, vpb.merge_options(4, P224, 5, assign))]
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
+    x = vpb.bf16_from_bits(x_bits)
+    modes = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
+    s = torch.zeros(1, 16, device="cuda")
+    vpb.vp_global_stack(dm, x, layers, None, modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    got = assign.cpu().numpy().astype(np.int64)
+    row_of, dst_tok = oracle.destinations(N, P224, 5, 4)
+    _, infos = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w)],
+                                   merge=[{"stride": 4, "tokens_per_view": P224, "patch_start": 5}],
+                                   assign=[got])
+    scores = infos[0]["merge"]["scores"]
+    # canonical row of each merged row: a view-2 destination's twin is the view-0 token at the
+    # same position, whose merged row is that position
+    tok = dst_tok
+    canon = np.where(tok // P224 == 2, tok % P224, np.arange(len(tok)))
+    src = np.nonzero(row_of < 0)[0]
+    n_ties = 0
+    for i in src:
+        sc = scores[i]
+        best = int(np.argmax(sc))
+        cls = canon == canon[best]
+        others = sc[~cls]
+        if sc[best] - others.max() <= 4e-2:
+            continue  # no clear winner: the bf16 metric decides, not the tie rule
+        want = int(np.nonzero(cls)[0].min())
+        assert got[i] == want, (int(i), int(got[i]), want)
+        n_ties += int(cls.sum() > 1)
+    assert n_ties >= 20, n_ties
