@@ -349,6 +349,18 @@ vp_status vp_router_noalloc(const vp_dims* dims, const vp_bf16* qkv, const vp_ro
 vp_status vp_profile_begin(int32_t max_launches);
 vp_status vp_profile_end(int32_t* n_launches, int32_t* launches, float* ms);
 
+/*
+ * Self-test of the bounded device waits (failure handling; not part of the method).
+ * Enqueues on `stream` one warp that waits on an mbarrier nothing arrives on, with a time
+ * limit of limit_ns nanoseconds instead of the kernels' 4 s, so that the wait gives up,
+ * sets VP_DEVERR_WAIT_TIMEOUT in the workspace's error word and returns, leaving the context
+ * usable; vp_read_device_error then reports VP_ERR_DEVICE_TIMEOUT.  The kernel runs for at
+ * least limit_ns.
+ *   ws, ws_bytes  any workspace of this library (its error word is the first 4 bytes; >= 256 B)
+ *   limit_ns      1e6 .. 2e9 (1 ms .. 2 s), else VP_ERR_INVALID_ARG before any launch
+ */
+vp_status vp_selftest_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

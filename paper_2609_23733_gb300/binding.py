@@ -9,7 +9,7 @@ from __future__ import annotations
 
 import ctypes
 import os
-from ctypes import POINTER, Structure, c_char_p, c_float, c_int32, c_size_t, c_uint32, c_void_p
+from ctypes import POINTER, Structure, c_char_p, c_float, c_int32, c_int64, c_size_t, c_uint32, c_void_p
 
 import numpy as np
 import torch
@@ -73,6 +73,7 @@ _SIGS = [
     ("vp_status_string", c_char_p, [c_int32]),
     ("vp_workspace_size", c_int32, [POINTER(VpDims), c_int32, POINTER(c_size_t)]),
     ("vp_read_device_error", c_int32, [c_void_p, c_size_t, POINTER(c_uint32), c_void_p]),
+    ("vp_selftest_wait_timeout", c_int32, [c_void_p, c_size_t, c_int64, c_void_p]),
     ("vp_router", c_int32, [POINTER(VpDims), c_void_p, POINTER(VpRouterWeights), c_void_p, c_void_p,
                             c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
                             c_void_p]),
@@ -235,6 +236,13 @@ def vp_workspace_size(dm: VpDims, what: int) -> int:
 def workspace(dm: VpDims, what: int, device="cuda") -> torch.Tensor:
     """A zeroed device workspace of the size the library asks for."""
     return torch.zeros(vp_workspace_size(dm, what), dtype=torch.uint8, device=device)
+
+
+def vp_selftest_wait_timeout(ws: torch.Tensor, limit_ns: int, stream=None):
+    """Enqueues the library's bounded-wait self-test: a wait that nothing satisfies gives up
+    after limit_ns and sets the timeout bit of ws's error word."""
+    _check(lib().vp_selftest_wait_timeout(_p(ws), ws.numel(), int(limit_ns), _stream(stream)),
+           "vp_selftest_wait_timeout")
 
 
 def vp_read_device_error(ws: torch.Tensor, stream=None) -> int:

@@ -480,6 +480,15 @@ vp_status vp_read_device_error(void* ws, size_t ws_bytes, uint32_t* host_bits, v
   return (bits & VP_DEVERR_WAIT_TIMEOUT) ? VP_ERR_DEVICE_TIMEOUT : VP_OK;
 }
 
+vp_status vp_selftest_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
+  if (!ws || ws_bytes < 256 || !aligned16(ws)) return VP_ERR_INVALID_ARG;
+  if (limit_ns < 1000000 || limit_ns > 2000000000) return VP_ERR_INVALID_ARG;
+  VP_TRY(check_device());
+  return from_cuda(launch_wait_selftest(static_cast<unsigned int*>(ws),
+                                        (unsigned long long)limit_ns,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
 vp_status vp_router(const vp_dims* dims, const vp_bf16* qkv, const vp_router_weights* rw,
                     const int32_t* force_modes, float* s, int32_t* modes, float* q_pool,
                     float* ctx, float* mean_v, float* r, void* ws, size_t ws_bytes, void* stream) {

@@ -74,11 +74,12 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Waits until the phase with the given parity has completed.  Gives up after
-// kWaitLimitNs, records VP_DEVERR_WAIT_TIMEOUT in *err and sets *abort_flag; returns
-// false in that case.  Returns immediately (false) if *abort_flag is already set.
+// Waits until the phase with the given parity has completed.  Gives up after limit_ns,
+// records VP_DEVERR_WAIT_TIMEOUT in *err and sets *abort_flag; returns false in that case.
+// Returns immediately (false) if *abort_flag is already set.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned int* err,
-                                          volatile int* abort_flag) {
+                                          volatile int* abort_flag,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_test_wait(bar, parity)) return true;  // already complete: no suspension
   // The time limit runs from the first check (after 255 unsuccessful tries), so that the
   // common short wait reads no clock.
@@ -90,7 +91,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsign
       const unsigned long long now = global_timer_ns();
       if (t0 == 0) {
         t0 = now;
-      } else if (now - t0 > kWaitLimitNs) {
+      } else if (now - t0 > limit_ns) {
         atomicOr(err, VP_DEVERR_WAIT_TIMEOUT);
         *abort_flag = 1;
         return false;
@@ -102,8 +103,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsign
 // mbar_wait for a converged warp: every lane polls, and the result is the same on every lane
 // (TMEM accesses and elected-lane issue after it are warp-collective).
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, unsigned int* err,
-                                               volatile int* abort_flag) {
-  const bool ok = mbar_wait(bar, parity, err, abort_flag);
+                                               volatile int* abort_flag,
+                                               unsigned long long limit_ns = kWaitLimitNs) {
+  const bool ok = mbar_wait(bar, parity, err, abort_flag, limit_ns);
   return __all_sync(0xffffffffu, ok);
 }
 

@@ -199,6 +199,10 @@ cudaError_t launch_unmerge_ln(int N, int D, const int* assign, const __nv_bfloat
                               const float* ls, const float* g, const float* b, float eps,
                               __nv_bfloat16* x, __nv_bfloat16* z, cudaStream_t st);
 
+// One warp waiting on an mbarrier that never completes, bounded by limit_ns (self-test of the
+// wait limit; sets VP_DEVERR_WAIT_TIMEOUT in *err).
+cudaError_t launch_wait_selftest(unsigned int* err, unsigned long long limit_ns, cudaStream_t st);
+
 cudaError_t launch_layer_norm(int M, int D, const __nv_bfloat16* x, const float* g,
                               const float* b, float eps, __nv_bfloat16* out, cudaStream_t st);
 

@@ -476,7 +476,28 @@ __global__ void bin_heads_kernel(int H, int N, const int32_t* modes, int32_t* he
   }
 }
 
+// Self-test of the bounded waits (failure handling, not the method): one warp waits on an
+// mbarrier that nothing ever arrives on, so the wait must give up after limit_ns, record
+// VP_DEVERR_WAIT_TIMEOUT and return.
+__global__ void wait_selftest_kernel(unsigned int* err, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbarrier_init();
+  }
+  __syncthreads();
+  mbar_wait_warp(&bar, 0, err, &abort_flag, limit_ns);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(unsigned int* err, unsigned long long limit_ns,
+                                 cudaStream_t st) {
+  wait_selftest_kernel<<<1, 32, 0, st>>>(err, limit_ns);
+  return cudaGetLastError();
+}
 
 size_t router_scratch_bytes(int H) {
   (void)H;

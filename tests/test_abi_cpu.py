@@ -209,3 +209,13 @@ def test_weight_structs_keep_their_tensors(vp):
     assert built["surrogate"].d2_b == int(refs["surrogate"]())
     assert built["qk"].q_norm_g == int(refs["qk"]())
     assert built["merge"].assign_out == 1 << 30
+
+
+def test_wait_selftest_validated_on_the_host(vp):
+    lib = vp.lib()
+    buf = (ctypes.c_uint8 * 4096)()
+    A = ctypes.c_void_p(((ctypes.addressof(buf) + 255) // 256) * 256)
+    for limit in (0, 999_999, 2_000_000_001, -5):  # outside 1 ms .. 2 s
+        assert lib.vp_selftest_wait_timeout(A, 1024, limit, None) == 1
+    assert lib.vp_selftest_wait_timeout(None, 1024, 50_000_000, None) == 1
+    assert lib.vp_selftest_wait_timeout(A, 128, 50_000_000, None) == 1  # no room for the error word
