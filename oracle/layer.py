@@ -139,19 +139,18 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
 
     Storage points (materialize, bf16): QKV, Y, Z~, the FFN hidden layer and the residual
     stream X_attn, X'.  The LN1 output X~ is not stored: the block feeds it straight into
-    the QKV projection.
+    the QKV projection, or, with merging, into the key metric and the merged tokens.
 
     merge: token merging around the attention (oracle.merge; a dict with stride,
-    tokens_per_view, patch_start): X~ (stored) is merged, the routed attention and W_O (+ b_O,
-    stored) run on the merged tokens, and every token adds LS1 times its merged token's
-    output.  assign: the merged row of every token to use instead of the oracle's matching
-    (the library's choice, for parity downstream of a near-tie)."""
+    tokens_per_view, patch_start): X~ is merged (the merged tokens are stored), the routed
+    attention and W_O (+ b_O, stored) run on the merged tokens, and every token adds LS1 times
+    its merged token's output.  assign: the merged row of every token to use instead of the
+    oracle's matching (the library's choice, for parity downstream of a near-tie)."""
     mat = materialize or _identity
     X = np.asarray(X, np.float64)
     Xt = layer_norm(X, lw["ln1_g"], lw["ln1_b"], eps)
     merged = None
     if merge is not None:
-        Xt = mat(Xt)
         row_of, dst_tok = destinations(X.shape[0], merge["tokens_per_view"], merge["patch_start"],
                                        merge["stride"])
         own, scores = match(key_metric(Xt, lw, mat), row_of, dst_tok)

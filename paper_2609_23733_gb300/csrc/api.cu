@@ -715,12 +715,14 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     float* sa_l = s_attn_out ? s_attn_out + (size_t)l * dims->H : nullptr;
     int32_t* m_l = modes_out ? modes_out + (size_t)l * dims->H : nullptr;
     if (w.merge) {
-      // (1) X~ = LN1(X); merge X~ (vp_merge_options); (2)-(3) routed attention of the merged
-      // tokens; unmerge: X_i += LS1 (.) A[merged row of i]
-      VP_TRY(from_cuda(launch_layer_norm(dims->N, D, x, w.ln1_g, w.ln1_b, ln_eps, zt, st)));
+      // (1) X~ = LN1(X), folded into the key metric and the merged tokens (not stored); merge
+      // X~ (vp_merge_options); (2)-(3) routed attention of the merged tokens; unmerge:
+      // X_i += LS1 (.) A[merged row of i].  The folded metric weights use the QKV fold's
+      // scratch, which merged blocks do not need.
       const MergeGeo g = make_merge_geo(dims->N, w.merge->tokens_per_view, w.merge->patch_start,
                                         w.merge->stride);
-      VP_TRY(from_cuda(launch_merge_prepare(g, dims->H, zt,
+      const MergeLn mln{part, w.ln1_g, w.ln1_b, ln_eps, wq, cq, bq};
+      VP_TRY(from_cuda(launch_merge_prepare(g, dims->H, x, mln,
                                             reinterpret_cast<const __nv_bfloat16*>(w.w_qkv),
                                             w.b_qkv, ms, sms, st)));
       if (w.merge->assign_out)

@@ -189,10 +189,22 @@ struct MergeScratch {
   __nv_bfloat16* xm;     // [Np][D] merged tokens
   unsigned int* err;
 };
-// x~ [N][D] -> s.assign, s.dst_tok, s.xm (D = 64 H, D % 256 == 0).
-cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* xt,
-                                 const __nv_bfloat16* w_qkv, const float* b_qkv,
-                                 const MergeScratch& s, int num_sms, cudaStream_t st);
+// LN1 of the merging, folded (its output is never stored): the row statistics of x and the
+// scratch of the folded metric weights.
+struct MergeLn {
+  const float2* part;        // [N][D / 128] (mean, M2) of x's 128-column blocks
+  const float* g;            // [D] LN1 gamma
+  const float* b;            // [D] LN1 beta
+  float eps;
+  __nv_bfloat16* w_fold;     // [64][D] head-mean key weights with gamma folded in
+  float* c_fold;             // [64] their row sums
+  float* b_fold;             // [64] folded bias
+};
+// x [N][D] (the block's input) -> s.assign, s.dst_tok, s.xm (D = 64 H, D % 256 == 0).
+cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* x,
+                                 const MergeLn& ln, const __nv_bfloat16* w_qkv,
+                                 const float* b_qkv, const MergeScratch& s, int num_sms,
+                                 cudaStream_t st);
 // x[i] = bf16(x[i] + ls (.) a[assign[i]]) and z[i] = LN(x[i]) (g, b, eps) over N rows of D
 // channels.
 cudaError_t launch_unmerge_ln(int N, int D, const int* assign, const __nv_bfloat16* a,

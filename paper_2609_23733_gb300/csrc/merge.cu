@@ -431,12 +431,16 @@ __global__ void merge_fill_kernel(int N, const int* assign, const int* offs, int
   members[offs[r] + atomicAdd(fill + r, 1)] = i;
 }
 
-// One warp per merged token: the fp32 mean of its members' rows of x~ (D = 256 C; lane l
-// holds 16-byte chunks c 32 + l).
+// One warp per merged token: the mean of its members' rows of LN1(x), normalised on the fly
+// (the LN1 output is not stored): for each member, its mean and 1 / sqrt(var + eps) from the
+// (mean, M2) of its 128-column blocks, then (x - mu) rstd summed in fp32; at the end
+// gamma (.) sum / count + beta (D = 256 C; lane l holds 16-byte chunks c 32 + l).
 template <int C>
-__global__ void __launch_bounds__(256, C <= 4 ? 3 : 1) merge_mean_kernel(int Np, const __nv_bfloat16* xt, const int* offs,
-                                  const int* members, __nv_bfloat16* xm) {
-  constexpr int D = 256 * C;
+__global__ void __launch_bounds__(256, C <= 4 ? 3 : 1)
+    merge_mean_kernel(int Np, const __nv_bfloat16* x, const float2* part, const float* gamma,
+                      const float* beta, float eps, const int* offs, const int* members,
+                      __nv_bfloat16* xm) {
+  constexpr int D = 256 * C, NB = D / 128;  // 128-column blocks of a row (NB <= 32)
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (r >= Np) return;
@@ -446,42 +450,63 @@ __global__ void __launch_bounds__(256, C <= 4 ? 3 : 1) merge_mean_kernel(int Np,
   for (int c = 0; c < C; ++c)
 #pragma unroll
     for (int k = 0; k < 8; ++k) acc[c][k] = 0.f;
-  // Member indices 32 at a time (one coalesced load), then their rows, two in flight.
+  // Member indices 32 at a time (one coalesced load), then their rows and statistics, two
+  // members in flight.
   for (int q0 = b; q0 < e; q0 += 32) {
     const int mine = q0 + lane < e ? members[q0 + lane] : 0;
     const int nm = min(32, e - q0);
     for (int k = 0; k < nm; k += 2) {  // two rows' loads issued before any arithmetic
       uint4 u[2][C];
+      float2 ps[2];
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
         const int i = __shfl_sync(0xffffffffu, mine, min(k + j, nm - 1));
 #pragma unroll
         for (int c = 0; c < C; ++c)
-          u[j][c] = k + j < nm ? __ldg(reinterpret_cast<const uint4*>(xt + (size_t)i * D + (c * 32 + lane) * 8))
-                               : make_uint4(0u, 0u, 0u, 0u);
+          u[j][c] = __ldg(reinterpret_cast<const uint4*>(x + (size_t)i * D + (c * 32 + lane) * 8));
+        ps[j] = lane < NB ? __ldg(part + (size_t)i * NB + lane) : make_float2(0.f, 0.f);
       }
 #pragma unroll
-      for (int j = 0; j < 2; ++j)
+      for (int j = 0; j < 2; ++j) {
+        if (k + j >= nm) break;  // uniform across the warp
+        float sm = ps[j].x;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+        const float mu = sm / (float)NB;
+        const float d = ps[j].x - mu;
+        float m2 = lane < NB ? ps[j].y + 128.f * d * d : 0.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m2 += __shfl_xor_sync(0xffffffffu, m2, o);
+        const float rstd = rsqrtf(m2 / (float)D + eps);
+        const float nmr = -mu * rstd;
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t w[4] = {u[j][c].x, u[j][c].y, u[j][c].z, u[j][c].w};
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {
-            acc[c][2 * kk] += bf16_lo(w[kk]);
-            acc[c][2 * kk + 1] += bf16_hi(w[kk]);
+            acc[c][2 * kk] += fmaf(bf16_lo(w[kk]), rstd, nmr);
+            acc[c][2 * kk + 1] += fmaf(bf16_hi(w[kk]), rstd, nmr);
           }
         }
+      }
     }
   }
   const float inv = 1.f / (float)(e - b);
 #pragma unroll
   for (int c = 0; c < C; ++c) {
+    const int col = (c * 32 + lane) * 8;
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gamma + col));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gamma + col) + 1);
+    const float4 b0 = __ldg(reinterpret_cast<const float4*>(beta + col));
+    const float4 b1 = __ldg(reinterpret_cast<const float4*>(beta + col) + 1);
+    const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
     uint4 o;
-    o.x = pack_bf16x2(acc[c][0] * inv, acc[c][1] * inv);
-    o.y = pack_bf16x2(acc[c][2] * inv, acc[c][3] * inv);
-    o.z = pack_bf16x2(acc[c][4] * inv, acc[c][5] * inv);
-    o.w = pack_bf16x2(acc[c][6] * inv, acc[c][7] * inv);
-    *reinterpret_cast<uint4*>(xm + (size_t)r * D + (c * 32 + lane) * 8) = o;
+    o.x = pack_bf16x2(fmaf(gg[0], acc[c][0] * inv, bb[0]), fmaf(gg[1], acc[c][1] * inv, bb[1]));
+    o.y = pack_bf16x2(fmaf(gg[2], acc[c][2] * inv, bb[2]), fmaf(gg[3], acc[c][3] * inv, bb[3]));
+    o.z = pack_bf16x2(fmaf(gg[4], acc[c][4] * inv, bb[4]), fmaf(gg[5], acc[c][5] * inv, bb[5]));
+    o.w = pack_bf16x2(fmaf(gg[6], acc[c][6] * inv, bb[6]), fmaf(gg[7], acc[c][7] * inv, bb[7]));
+    *reinterpret_cast<uint4*>(xm + (size_t)r * D + col) = o;
   }
 }
 
@@ -575,22 +600,30 @@ MergeGeo make_merge_geo(int N, int P, int ps, int stride) {
   return g;
 }
 
-cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* xt,
-                                 const __nv_bfloat16* w_qkv, const float* b_qkv,
-                                 const MergeScratch& s, int num_sms, cudaStream_t st) {
+cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* x,
+                                 const MergeLn& ln, const __nv_bfloat16* w_qkv,
+                                 const float* b_qkv, const MergeScratch& s, int num_sms,
+                                 cudaStream_t st) {
   const int D = 64 * H;
   prof_before(VP_KERNEL_MERGE, st);
   metric_weights_kernel<<<(64 * D + 255) / 256, 256, 0, st>>>(w_qkv, b_qkv, H, D, s.wbar, s.bbar);
   prof_after(st);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  // The metric of LN1(x) with LN1 folded into its weights, as in the QKV projection.
+  if ((e = launch_ln_fold_weights(64, D, s.wbar, ln.g, ln.b, s.bbar, ln.w_fold, ln.c_fold,
+                                  ln.b_fold, st)) != cudaSuccess)
+    return e;
   LinearArgs la{};
   la.M = g.N;
   la.N = 64;
   la.K = D;
-  la.A = xt;
-  la.W = s.wbar;
-  la.bias = s.bbar;
+  la.A = x;
+  la.W = ln.w_fold;
+  la.bias = ln.b_fold;
+  la.ln_part = ln.part;
+  la.ln_c = ln.c_fold;
+  la.ln_eps = ln.eps;
   la.act = VP_ACT_NONE;
   la.out = s.kbar;
   la.err = s.err;
@@ -636,12 +669,13 @@ cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* 
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   prof_before(VP_KERNEL_MERGE, st);
+  const int grid = (g.Np + 7) / 8;
   switch (D / 256) {
-    case 1: merge_mean_kernel<1><<<(g.Np + 7) / 8, 256, 0, st>>>(g.Np, xt, s.offs, s.members, s.xm); break;
-    case 2: merge_mean_kernel<2><<<(g.Np + 7) / 8, 256, 0, st>>>(g.Np, xt, s.offs, s.members, s.xm); break;
-    case 3: merge_mean_kernel<3><<<(g.Np + 7) / 8, 256, 0, st>>>(g.Np, xt, s.offs, s.members, s.xm); break;
-    case 4: merge_mean_kernel<4><<<(g.Np + 7) / 8, 256, 0, st>>>(g.Np, xt, s.offs, s.members, s.xm); break;
-    case 8: merge_mean_kernel<8><<<(g.Np + 7) / 8, 256, 0, st>>>(g.Np, xt, s.offs, s.members, s.xm); break;
+    case 1: merge_mean_kernel<1><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
+    case 2: merge_mean_kernel<2><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
+    case 3: merge_mean_kernel<3><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
+    case 4: merge_mean_kernel<4><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
+    case 8: merge_mean_kernel<8><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
     default: prof_after(st); return cudaErrorInvalidValue;
   }
   prof_after(st);
