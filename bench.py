@@ -386,6 +386,8 @@ def run_ours(args):
         line["qkv_positional"] = qk_probe(vpb, dev, N, dws[0])
     if args.tome:
         line["token_merging_s100"] = tome_probe(vpb, dev, N, dws, fm)
+    if args.mix:
+        line["mix_sweep_s64"] = mix_probe(vpb, dev, pk)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
@@ -535,6 +537,55 @@ def qk_probe(vpb, dev, N, dw):
         res[f"gemm_ms_{name}"] = ms["gemm"] / 5
     res["qk_epilogue_ms"] = res["gemm_ms_qk_norm_rope"] - res["gemm_ms_plain"]
     return res
+
+
+def mix_probe(vpb, dev, pk, steps=3, warmup=2):
+    """The routing-mix sweep: one layer (QKV, router, heads, W_O) at S=64 views (518 px,
+    87,936 tokens) with 0 / 25 / 50 / 100 % of the heads forced to full mode and the rest
+    spread over the cheaper modes; layer time per mix, the attention launch's share, and a
+    straight-line fit of the layer time against the number of full heads."""
+    import torch
+    wl = synth.WORKLOADS["s64_mix_sweep"]
+    N = wl.N
+    dw = vpb.to_device(synth.make_layer_weights(synth.rng(wl.seed)), dev)
+    x = vpb.bf16_from_bits(synth.make_tokens(wl.seed, N), dev)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_LAYER, dev)
+    out = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+    modes = torch.zeros(H, dtype=torch.int32, device=dev)
+    rw, sw = vpb.router_weights(dw), vpb.surrogate_weights(dw)
+    peak = pk.get("bf16_tflops") or 1900.0
+    rows, n_full, t = [], [], []
+    for frac in (0.0, 0.25, 0.5, 1.0):
+        fm = torch.from_numpy(synth.forced_mix(H, frac)).to(dev)
+
+        def step():
+            vpb.vp_moh_global_attention(dm, x, dw["w_qkv"], dw["b_qkv"], dw["w_o"], dw["b_o"], rw, sw, fm, out,
+                                        None, None, None, modes, ws)
+
+        for _ in range(warmup):
+            step()
+        torch.cuda.synchronize()
+        vpb.vp_profile_begin(64 * steps)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            step()
+        b.record()
+        torch.cuda.synchronize()
+        _, cnt, cls_ms = vpb.vp_profile_end()
+        ms = a.elapsed_time(b) / steps
+        nf = int((modes.cpu().numpy() == synth.MODE_FULL).sum())
+        attn_ms = cls_ms["attn_full"] / steps
+        full_tf = 4.0 * N * N * d * nf / (attn_ms * 1e-3) / 1e12 if nf else None
+        rows.append({"full_fraction": frac, "full_heads": nf, "ms_per_layer": ms, "attn_ms": attn_ms,
+                     "attn_tflops": full_tf, "attn_frac_of_burst": full_tf / peak if nf else None})
+        n_full.append(nf)
+        t.append(ms)
+    slope, icpt = np.polyfit(np.array(n_full, float), np.array(t), 1)
+    return {"workload": wl.name, "views": wl.views, "tokens": N, "layers": 1, "mixes": rows,
+            "fit_ms": {"per_full_head": float(slope), "fixed": float(icpt)},
+            "speedup_vs_all_full": {f"{r['full_fraction']:.2f}": t[-1] / r["ms_per_layer"] for r in rows}}
 
 
 def full_attention_probe(vpb, dev, N, dw, pk):
@@ -694,6 +745,7 @@ def main():
     ap.add_argument("--no-variants", dest="variants", action="store_false")
     ap.add_argument("--no-qk", dest="qk", action="store_false")
     ap.add_argument("--no-tome", dest="tome", action="store_false")
+    ap.add_argument("--no-mix", dest="mix", action="store_false", help="skip the S=64 routing-mix sweep")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
                                               "surrogate", "mean", "bin", "merge"],
                     default=None,
