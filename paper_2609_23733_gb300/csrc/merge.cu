@@ -103,7 +103,8 @@ __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_b
 //               of two 256-column fp32 accumulators (the epilogue of one chunk overlaps the
 //               MMAs of the next);
 //   warps 4-19  argmax: a source row (TMEM lane) and a quarter of each chunk's columns per
-//               thread, 32 columns (a piece) per tcgen05.ld, the next in flight.  A tree gives
+//               thread, loaded into registers (two tcgen05.ld of 32 columns) before the
+//               accumulator is released, so that the max trees overlap the next MMAs.  A tree gives
 //               the piece's max; a piece whose max beats the row's best is copied to the
 //               thread's slot in shared memory, and the column is looked up there once, at the
 //               end of the segment.  Chunks ascend within a segment, so the first piece that
@@ -289,13 +290,17 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
         tc_fence_after();
         const int c0 = ch * kMatchN + part * kCols;  // first destination of the part
         const int valid = g.Np - c0;                 // columns past it hold no destination
-        float v[2][32];
-        tmem_ld32(t_lane + ab * kMatchN, v[0]);
+        // Both pieces into registers, then the accumulator goes back to the MMA warp at once:
+        // the max trees below overlap the next chunks' MMAs.
+        float v[kCols / 32][32];
+#pragma unroll
+        for (int p = 0; p < kCols / 32; ++p) tmem_ld32(t_lane + ab * kMatchN + 32 * p, v[p]);
         tmem_wait_ld();
+        tc_fence_before();
+        mbar_arrive(&sm.acc_empty[ab]);
 #pragma unroll
         for (int p = 0; p < kCols / 32; ++p) {
-          if (p + 1 < kCols / 32) tmem_ld32(t_lane + ab * kMatchN + 32 * (p + 1), v[(p + 1) & 1]);
-          float* x = v[p & 1];
+          float* x = v[p];
           if (32 * p + 32 > valid) {
 #pragma unroll
             for (int k = 0; k < 32; ++k)
@@ -316,10 +321,7 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
             for (int j = 0; j < 8; ++j)
               slot[(j + lane) & 7] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
           }
-          tmem_wait_ld();
         }
-        tc_fence_before();
-        mbar_arrive(&sm.acc_empty[ab]);
       }
       if (!ok) break;
       u += sg.c1 - sg.c0;
