@@ -1,11 +1,12 @@
 // Router of VGGT-Prime (§4.1) and routing (§4.2) on sm_103a.
 //
 // Two sweeps over the token axis, both split across CTAs with online-softmax partials:
-//   router_pool_kernel  (§4.1, pooling): e_i = w_h^T (tanh(W_h q_i + bW) (.) sigma(U_h q_i + bU))
-//       The [16 tokens x 64] x [64 x 128] projection onto [W_h; U_h] runs on the tensor
-//       cores (mma.sync m16n8k16, fp32 accumulation); each warp keeps a running
-//       (max, sum, sum p q) of alpha's softmax, the last CTA of a head combines the
-//       partials into q_pool = sum_i alpha_i q_i.
+//   router_pool_tc_kernel  (§4.1, pooling): e_i = w_h^T (tanh(W_h q_i + bW) (.) sigma(U_h q_i + bU))
+//       The [128 tokens x 64] x [64 x 128] projection onto [W_h; U_h] runs on the
+//       tcgen05 tensor cores (TMA-fed shared-memory operands, fp32 accumulators in TMEM);
+//       each token thread keeps a running (max, sum, sum p q) of alpha's softmax, the CTA
+//       merges them, and the last CTA of a head combines the partials into
+//       q_pool = sum_i alpha_i q_i.
 //   router_keys_kernel  (§4.1 routing attention + §4.3 context + mean of V):
 //       l_j = beta_h / sqrt(d) * q_pool . k_j; running (max, sum 2^(l-max), sum p v, sum v)
 //       per CTA; the last CTA of a head derives s_h = max_j r_h(j) = 1 / sum_j e^(l_j - max),
@@ -21,18 +22,7 @@ namespace vp {
 
 namespace {
 
-constexpr int kPoolThreads = 128;
 constexpr int kKeyThreads = 256;
-constexpr int kBStride = 72;  // padded smem row (bf16 elements): 144 bytes, conflict-free
-
-__device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, uint32_t b0,
-                                               uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 
 // tanh(x) * sigma(y) for the pooling logits of §4.1, two at a time on packed f32x2 pairs, in a
 // form that needs no clamps:
@@ -61,164 +51,12 @@ __device__ __forceinline__ void token_range(int N, int n_split, int split, int a
   t1 = min(N, t0 + per);
 }
 
-// ------------------------------------------------------------------ pooling sweep
-__global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a, RouterScratch sc,
-                                                                    int n_split) {
-  const int h = blockIdx.y, split = blockIdx.x;
-  const int N = a.N, H = a.H;
-  const size_t row_pitch = (size_t)3 * H * kHeadDim;  // elements between consecutive tokens
-  const bool mean_pool = (a.variant & VP_VARIANT_MEAN_QPOOL) != 0;  // §5 component ablation
-
-  __shared__ __align__(16) __nv_bfloat16 sB[128 * kBStride];  // rows 0..63 W_h, 64..127 U_h
-  __shared__ __align__(16) float s_bias[128];                // bW | bU
-  __shared__ __align__(16) float s_w[64];
-  __shared__ float s_part[4][kPoolPartial];
-
-  const int tid = threadIdx.x;
-  // Stage [W_h; U_h] (128 rows x 128 bytes) in padded rows.
-  for (int i = tid; i < 128 * 8; i += kPoolThreads) {
-    const int row = i >> 3, ch = i & 7;
-    const __nv_bfloat16* src = (row < 64 ? a.W : a.U) + ((size_t)h * 64 + (row & 63)) * 64 + ch * 8;
-    *reinterpret_cast<uint4*>(&sB[row * kBStride + ch * 8]) = *reinterpret_cast<const uint4*>(src);
-  }
-  if (tid < 64) {
-    s_bias[tid] = a.bW ? a.bW[h * 64 + tid] : 0.f;
-    s_bias[64 + tid] = a.bU ? a.bU[h * 64 + tid] : 0.f;
-    s_w[tid] = __bfloat162float(a.w[h * 64 + tid]);
-  }
-  __syncthreads();
-
-  int t0, t1;
-  token_range(N, n_split, split, 16, t0, t1);
-  const int warp = tid >> 5, lane = tid & 31;
-  const int r = lane >> 2, c = lane & 3;
-  const __nv_bfloat16* qbase = a.qkv + (size_t)h * kHeadDim + 16 * c;
-
-  float M = -INFINITY, lsum = 0.f;
-  float accq[16];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) accq[i] = 0.f;
-
-  // Each thread holds channels 16c..16c+15 of rows ra and rb.  The MMA's reduction index k
-  // is permuted consistently in A and B (logical k pair (kk, 2c) <-> channels 16c + 4kk +
-  // {0,1}, pair (kk, 2c + 8) <-> 16c + 4kk + {2,3}), so that every thread reads 32 contiguous
-  // bytes of its rows and of the weight rows.  The next tile's rows are loaded while the
-  // current tile is computed.
-  auto load_rows = [&](int base, uint4& x0, uint4& x1, uint4& y0, uint4& y1) {
-    const int ra = base + r, rb = base + r + 8;
-    const uint4* pa = reinterpret_cast<const uint4*>(qbase + (size_t)(ra < t1 ? ra : t0) * row_pitch);
-    const uint4* pb = reinterpret_cast<const uint4*>(qbase + (size_t)(rb < t1 ? rb : t0) * row_pitch);
-    x0 = __ldg(pa);
-    x1 = __ldg(pa + 1);
-    y0 = __ldg(pb);
-    y1 = __ldg(pb + 1);
-  };
-  uint4 nx0, nx1, ny0, ny1;
-  if (t0 + 16 * warp < t1) load_rows(t0 + 16 * warp, nx0, nx1, ny0, ny1);
-  for (int base = t0 + 16 * warp; base < t1; base += 64) {
-    const int ra = base + r, rb = base + r + 8;
-    const bool va = ra < t1, vb = rb < t1;
-    uint32_t qa[8], qb[8];
-    {
-      const uint4 x0 = nx0, x1 = nx1, y0 = ny0, y1 = ny1;
-      if (base + 64 < t1) load_rows(base + 64, nx0, nx1, ny0, ny1);
-      qa[0] = x0.x; qa[1] = x0.y; qa[2] = x0.z; qa[3] = x0.w;
-      qa[4] = x1.x; qa[5] = x1.y; qa[6] = x1.z; qa[7] = x1.w;
-      qb[0] = y0.x; qb[1] = y0.y; qb[2] = y0.z; qb[3] = y0.w;
-      qb[4] = y1.x; qb[5] = y1.y; qb[6] = y1.z; qb[7] = y1.w;
-    }
-    // Pooling logits (both 0 under the mean-pooling ablation: alpha = 1/N exactly).
-    float ea = 0.f, eb = 0.f;
-    if (!mean_pool) {
-    float acc[16][4];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
-      const uint4* pw = reinterpret_cast<const uint4*>(&sB[(8 * j + r) * kBStride + 16 * c]);
-      const uint4 w0 = pw[0], w1 = pw[1];
-      const uint32_t bw[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        const uint32_t af[4] = {qa[2 * kk], qb[2 * kk], qa[2 * kk + 1], qb[2 * kk + 1]};
-        mma_bf16_16816(acc[j], af, bw[2 * kk], bw[2 * kk + 1]);
-      }
-    }
-    // Pooling logits: columns 8j + 2c + e of the W half (j < 8) pair with the same
-    // columns of the U half (j + 8) in the same thread; the two columns e = 0, 1 of a row
-    // form one packed pair.
-    float2 pa = make_float2(0.f, 0.f), pb = make_float2(0.f, 0.f);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int l = 8 * j + 2 * c;
-      const float2 bw = *reinterpret_cast<const float2*>(&s_bias[l]);
-      const float2 bu = *reinterpret_cast<const float2*>(&s_bias[64 + l]);
-      const float2 wl = *reinterpret_cast<const float2*>(&s_w[l]);
-      pa = ffma2(wl, tanh_times_sigmoid2(fadd2(make_float2(acc[j][0], acc[j][1]), bw),
-                                         fadd2(make_float2(acc[j + 8][0], acc[j + 8][1]), bu)), pa);
-      pb = ffma2(wl, tanh_times_sigmoid2(fadd2(make_float2(acc[j][2], acc[j][3]), bw),
-                                         fadd2(make_float2(acc[j + 8][2], acc[j + 8][3]), bu)), pb);
-    }
-    ea = pa.x + pa.y;
-    eb = pb.x + pb.y;
-    ea += __shfl_xor_sync(0xffffffffu, ea, 1);
-    ea += __shfl_xor_sync(0xffffffffu, ea, 2);
-    eb += __shfl_xor_sync(0xffffffffu, eb, 1);
-    eb += __shfl_xor_sync(0xffffffffu, eb, 2);
-    }
-    if (!va) ea = -INFINITY;
-    if (!vb) eb = -INFINITY;
-    float mc = fmaxf(ea, eb);
-    mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, 4));
-    mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, 8));
-    mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, 16));
-    if (mc == -INFINITY) continue;  // warp-uniform
-    const float Mn = fmaxf(M, mc);
-    const float scale = __expf(M - Mn);  // 0 when M = -inf
-    const float pa = __expf(ea - Mn), pb = __expf(eb - Mn);
-    lsum = lsum * scale + (pa + pb);
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {
-      accq[2 * m] = accq[2 * m] * scale + pa * bf16_lo(qa[m]) + pb * bf16_lo(qb[m]);
-      accq[2 * m + 1] = accq[2 * m + 1] * scale + pa * bf16_hi(qa[m]) + pb * bf16_hi(qb[m]);
-    }
-    M = Mn;
-  }
-  // Reduce over the 8 row groups (lane bits 2..4); M is warp-uniform.
-#pragma unroll
-  for (int o = 4; o < 32; o <<= 1) {
-    lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
-#pragma unroll
-    for (int i = 0; i < 16; ++i) accq[i] += __shfl_xor_sync(0xffffffffu, accq[i], o);
-  }
-  if (lane < 4) {
-#pragma unroll
-    for (int i = 0; i < 16; ++i) s_part[warp][2 + 16 * c + i] = accq[i];
-    if (lane == 0) {
-      s_part[warp][0] = M;
-      s_part[warp][1] = lsum;
-    }
-  }
-  __syncthreads();
-  float* part = sc.pool_part + ((size_t)h * kPoolSplitMax + split) * kPoolPartial;
-  if (tid < 64) {
-    float Mx = -INFINITY;
-    for (int w = 0; w < 4; ++w) Mx = fmaxf(Mx, s_part[w][0]);
-    float acc = 0.f, l = 0.f;
-    if (Mx != -INFINITY) {
-      for (int w = 0; w < 4; ++w) {
-        const float f = __expf(s_part[w][0] - Mx);
-        acc += f * s_part[w][2 + tid];
-        l += f * s_part[w][1];
-      }
-    }
-    part[2 + tid] = acc;
-    if (tid == 0) {
-      part[0] = Mx;
-      part[1] = l;
-    }
-  }
-  // Last CTA of this head combines the partials into q_pool.
+// The last CTA of head h to publish its partial (max, sum, sum p q) combines the n_split
+// partials into q_pool.  Called by every thread of the CTA.
+__device__ __forceinline__ void pool_finish(const RouterArgs& a, const RouterScratch& sc, int h,
+                                            int n_split) {
   __shared__ int s_last;
+  const int tid = threadIdx.x;
   __threadfence();
   __syncthreads();
   if (tid == 0) s_last = (atomicAdd(&sc.counters[h], 1u) == (unsigned)(n_split - 1));
@@ -241,6 +79,254 @@ __global__ void __launch_bounds__(kPoolThreads) router_pool_kernel(RouterArgs a,
     sc.q_pool[h * 64 + tid] = q;
     if (a.q_pool_out) a.q_pool_out[h * 64 + tid] = q;
   }
+}
+
+// ------------------------------------------------------------------ pooling sweep (tcgen05)
+// The same sweep with the [W_h; U_h] projection on the 5th-generation tensor cores: a CTA
+// takes a run of 128-token tiles of one head.
+//   warp 4   TMA: [W_h; U_h] once (two 64 x 64 boxes into one 128-row, 128-byte-swizzled
+//            operand), then the tiles' Q rows (128 x 64, 16 KB) through a kPoolTcStages ring;
+//   warp 5   TMEM owner and MMA issue: four tcgen05.mma M128 N128 K16 per tile into one of
+//            two 128-column fp32 accumulators (columns 0-63: W_h q, 64-127: U_h q);
+//   warps 0-3  one token per thread (TMEM lane): the logit e = w_h . (tanh(W_h q + bW) (.)
+//            sigma(U_h q + bU)) from two halves of 32 + 32 accumulator columns, then a running
+//            softmax of its own tokens (max M, sum, sum p q over the 64 channels of its Q row,
+//            read from the shared-memory tile; rescaled only when M grows), released tile by
+//            tile; at the end the 128 threads' partials merge into the CTA's (max, sum,
+//            sum p q), which pool_finish combines over the CTAs of the head.
+constexpr int kPoolTcStages = 4;
+constexpr int kPoolTcThreads = 192;
+constexpr uint32_t kPoolTcTmemCols = 256;
+
+struct PoolTcSmem {
+  __nv_bfloat16 q[kPoolTcStages][128 * 64];
+  __nv_bfloat16 wu[128 * 64];
+  float bias[128];  // bW | bU
+  float wv[64];     // w_h
+  float red_m[4], red_l[4];
+  float red_acc[4][64];
+  uint64_t q_full[kPoolTcStages], q_empty[kPoolTcStages];
+  uint64_t wu_full, acc_full[2], acc_empty[2], drain;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__global__ void __launch_bounds__(kPoolTcThreads)
+    router_pool_tc_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                          const __grid_constant__ CUtensorMap tmap_w,
+                          const __grid_constant__ CUtensorMap tmap_u, RouterArgs a,
+                          RouterScratch sc, int n_split) {
+  extern __shared__ unsigned char smem_raw[];
+  PoolTcSmem& sm = *reinterpret_cast<PoolTcSmem*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int h = blockIdx.y, split = blockIdx.x;
+  const int N = a.N;
+  const int n_tiles_all = (N + 127) / 128;
+  const int tile0 = (int)((long long)split * n_tiles_all / n_split);
+  const int tile1 = (int)((long long)(split + 1) * n_tiles_all / n_split);
+  const int n_tiles = tile1 - tile0;  // >= 1 (n_split <= n_tiles_all)
+  const int tok_end = min(N, tile1 * 128);
+  const int tid = threadIdx.x;
+  const int warp = warp_uniform_id(), lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+  unsigned int* err = sc.err;
+
+  if (tid == 0) {
+    for (int s = 0; s < kPoolTcStages; ++s) {
+      mbar_init(&sm.q_full[s], 1);
+      mbar_init(&sm.q_empty[s], 128);
+    }
+    mbar_init(&sm.wu_full, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.acc_full[b], 1);
+      mbar_init(&sm.acc_empty[b], 128);
+    }
+    mbar_init(&sm.drain, 1);
+    sm.abort_flag = 0;
+    fence_mbarrier_init();
+    fence_proxy_async_smem();
+    tma_prefetch_desc(&tmap_q);
+  }
+  if (tid < 64) {
+    sm.bias[tid] = a.bW ? a.bW[h * 64 + tid] : 0.f;
+    sm.bias[64 + tid] = a.bU ? a.bU[h * 64 + tid] : 0.f;
+    sm.wv[tid] = __bfloat162float(a.w[h * 64 + tid]);
+  }
+  if (warp == 5) {
+    tmem_alloc(&sm.tmem_base, kPoolTcTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
+
+  float Mx = -INFINITY, lsum = 0.f;  // epilogue threads: this thread's tokens
+  float acc[64];
+#pragma unroll
+  for (int c = 0; c < 64; ++c) acc[c] = 0.f;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ TMA producer
+    bool ok = true;
+    if (elect_one()) {
+      mbar_arrive_expect_tx(&sm.wu_full, 128 * 64 * 2);
+      tma_load_2d(sm.wu, &tmap_w, &sm.wu_full, 0, h * 64);
+      tma_load_2d(sm.wu + 64 * 64, &tmap_u, &sm.wu_full, 0, h * 64);
+    }
+    __syncwarp();
+    int i = 0;
+    for (; i < n_tiles && ok; ++i) {
+      const int st = i % kPoolTcStages;
+      ok = mbar_wait_warp(&sm.q_empty[st], ((i / kPoolTcStages) & 1) ^ 1, err, abort_flag);
+      if (!ok) break;
+      if (elect_one()) {
+        mbar_arrive_expect_tx(&sm.q_full[st], 128 * 64 * 2);
+        tma_load_2d(sm.q[st], &tmap_q, &sm.q_full[st], h * 64, (tile0 + i) * 128);
+      }
+      __syncwarp();
+    }
+    if (!ok && lane == 0) {  // let issued copies land before the CTA releases its smem
+      for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.wu_full, 0); ++k) {}
+      for (int s = 0; s < kPoolTcStages; ++s) {
+        if (i > s) {
+          const int last = (i - 1 - s) / kPoolTcStages * kPoolTcStages + s;
+          for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.q_full[s], (last / kPoolTcStages) & 1); ++k) {}
+        }
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------ MMA issue
+    const uint32_t idesc = idesc_bf16(128, 128, 0, 0);
+    const uint64_t db = sdesc_sw128(smem_u32(sm.wu));
+    bool ok = mbar_wait_warp(&sm.wu_full, 0, err, abort_flag);
+    for (int i = 0; i < n_tiles && ok; ++i) {
+      const int st = i % kPoolTcStages, ab = i & 1;
+      ok = mbar_wait_warp(&sm.q_full[st], (i / kPoolTcStages) & 1, err, abort_flag) &&
+           mbar_wait_warp(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1, err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      const uint64_t da = sdesc_sw128(smem_u32(sm.q[st]));
+      if (elect_one()) {
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)  // K = 64 channels: 4 x K16, +32 bytes per step
+          tc_mma_ss(tmem + ab * 128, da + 2 * kk, db + 2 * kk, idesc, kk > 0 ? 1u : 0u);
+        tc_commit(&sm.acc_full[ab]);
+      }
+      __syncwarp();
+    }
+    if (!ok) {
+      if (elect_one()) {
+        tc_commit(&sm.drain);
+        for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.drain, 0); ++k) {}
+      }
+      __syncwarp();
+    }
+  } else {
+    // ------------------------------------------------------------ logits + running softmax
+    const int row = warp * 32 + lane;  // TMEM lane of this thread's token
+    const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
+    bool ok = true;
+    for (int i = 0; i < n_tiles && ok; ++i) {
+      const int st = i % kPoolTcStages, ab = i & 1;
+      ok = mbar_wait_warp(&sm.acc_full[ab], (i >> 1) & 1, err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      float e2x = 0.f, e2y = 0.f;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float zw[32], zu[32];
+        tmem_ld32(t_lane + ab * 128 + 32 * half, zw);
+        tmem_ld32(t_lane + ab * 128 + 64 + 32 * half, zu);
+        tmem_wait_ld();
+        if (half == 1) {  // the accumulator is in registers: back to the MMA warp
+          tc_fence_before();
+          mbar_arrive(&sm.acc_empty[ab]);
+        }
+        float2 pe = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const int l = 32 * half + 2 * k;
+          const float2 bw = *reinterpret_cast<const float2*>(&sm.bias[l]);
+          const float2 bu = *reinterpret_cast<const float2*>(&sm.bias[64 + l]);
+          const float2 wl = *reinterpret_cast<const float2*>(&sm.wv[l]);
+          pe = ffma2(wl, tanh_times_sigmoid2(fadd2(make_float2(zw[2 * k], zw[2 * k + 1]), bw),
+                                             fadd2(make_float2(zu[2 * k], zu[2 * k + 1]), bu)),
+                     pe);
+        }
+        e2x += pe.x;
+        e2y += pe.y;
+      }
+      const float e = (a.variant & VP_VARIANT_MEAN_QPOOL) ? 0.f : e2x + e2y;
+      const int tok = (tile0 + i) * 128 + row;
+      if (tok < tok_end) {
+        if (e > Mx) {  // the running maximum grows: rescale (exp(-inf) = 0 on the first token)
+          const float sc_ = __expf(Mx - e);
+          lsum *= sc_;
+#pragma unroll
+          for (int c = 0; c < 64; ++c) acc[c] *= sc_;
+          Mx = e;
+        }
+        const float p = __expf(e - Mx);
+        lsum += p;
+        const unsigned char* qrow = reinterpret_cast<const unsigned char*>(sm.q[st]) + row * 128;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {  // 16-byte chunk j of the row sits at chunk j ^ (row & 7)
+          const uint4 u = *reinterpret_cast<const uint4*>(qrow + ((j ^ (row & 7)) << 4));
+          const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            acc[8 * j + 2 * k] = fmaf(p, bf16_lo(w4[k]), acc[8 * j + 2 * k]);
+            acc[8 * j + 2 * k + 1] = fmaf(p, bf16_hi(w4[k]), acc[8 * j + 2 * k + 1]);
+          }
+        }
+      }
+      mbar_arrive(&sm.q_empty[st]);
+    }
+  }
+  // Merge the 128 token threads' partials: the CTA maximum, then scaled sums of l and sum p q.
+  if (warp < 4) {
+    float m = Mx;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if (lane == 0) sm.red_m[warp] = m;
+  }
+  __syncthreads();
+  const float M_cta = fmaxf(fmaxf(sm.red_m[0], sm.red_m[1]), fmaxf(sm.red_m[2], sm.red_m[3]));
+  if (warp < 4) {
+    const float f = Mx == -INFINITY ? 0.f : __expf(Mx - M_cta);
+    float l = lsum * f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+#pragma unroll
+    for (int c = 0; c < 64; ++c) {
+      float v = acc[c] * f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      acc[c] = v;
+    }
+    if (lane == 0) {
+      sm.red_l[warp] = l;
+#pragma unroll
+      for (int c = 0; c < 64; ++c) sm.red_acc[warp][c] = acc[c];
+    }
+  }
+  __syncthreads();
+  float* part = sc.pool_part + ((size_t)h * kPoolSplitMax + split) * kPoolPartial;
+  if (tid < 64) {
+    part[2 + tid] = sm.red_acc[0][tid] + sm.red_acc[1][tid] + sm.red_acc[2][tid] + sm.red_acc[3][tid];
+    if (tid == 0) {
+      part[0] = M_cta;
+      part[1] = sm.red_l[0] + sm.red_l[1] + sm.red_l[2] + sm.red_l[3];
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kPoolTcTmemCols);
+  }
+  pool_finish(a, sc, h, n_split);
 }
 
 // ------------------------------------------------------------------ key sweep
@@ -554,11 +640,24 @@ cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_
                           cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(sc.counters, 0, 512, st);
   if (e != cudaSuccess) return e;
-  // Enough CTAs to cover every SM a few times; at least 64 tokens per CTA.
-  int pool_split = (4 * num_sms + a.H - 1) / a.H;
-  pool_split = max(1, min(min(pool_split, kPoolSplitMax), (a.N + 63) / 64));
+  // Pooling sweep on the tensor cores: two CTAs per SM (TMEM 2 x 256 columns), runs of
+  // 128-token tiles.
+  const int n_tiles = (a.N + 127) / 128;
+  int pool_split = (2 * num_sms + a.H - 1) / a.H;
+  pool_split = max(1, min(min(pool_split, kPoolSplitMax), n_tiles));
+  CUtensorMap tq, tw, tu;  // Q rows of all heads, W and U as [H 64][64]; 128-byte swizzle
+  if ((e = make_tmap_bf16_2d(&tq, a.qkv, (uint64_t)3 * a.H * 64, (uint64_t)a.N,
+                             (uint64_t)3 * a.H * 64, 64, 128)) != cudaSuccess)
+    return e;
+  if ((e = make_tmap_bf16_2d(&tw, a.W, 64, (uint64_t)a.H * 64, 64, 64, 64)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16_2d(&tu, a.U, 64, (uint64_t)a.H * 64, 64, 64, 64)) != cudaSuccess) return e;
+  const int smem = (int)sizeof(PoolTcSmem) + 1024;
+  if ((e = cudaFuncSetAttribute(router_pool_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                smem)) != cudaSuccess)
+    return e;
   prof_before(VP_KERNEL_ROUTER_POOL, st);
-  router_pool_kernel<<<dim3(pool_split, a.H), kPoolThreads, 0, st>>>(a, sc, pool_split);
+  router_pool_tc_kernel<<<dim3(pool_split, a.H), kPoolTcThreads, smem, st>>>(tq, tw, tu, a, sc,
+                                                                            pool_split);
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
