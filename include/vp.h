@@ -303,22 +303,33 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
  * whose memory pool already reserves the GPU's memory and forbids raw cudaMalloc, or a
  * service that must not allocate once it is running).  The paper has no counterpart: this
  * is an interface choice of the library, not a step of the method.
- *   Arguments and outputs are those of vp_router, minus ws / ws_bytes; the results are the
- *   same.  The router's scratch comes from one fixed device buffer inside the library,
- *   large enough for up to 32 heads (about 1.56 MiB, held on every GPU that loads the
- *   library until the process exits); a call that would need more returns
- *   VP_ERR_STATIC_SCRATCH.  The call allocates nothing (no cudaMalloc, cudaFree or
- *   allocating library routine).
- *   The first call on a device looks up the buffer's device address (set-up, once per
- *   device, with that device current); make that first call before any stream capture.
+ *   Arguments, checks and outputs are those of vp_router, minus ws / ws_bytes (dims->variant
+ *   included; H outside 1..32 is VP_ERR_UNSUPPORTED_SHAPE); the results are the same.  The
+ *   router's scratch comes from one fixed device buffer inside the library, large enough for
+ *   up to 32 heads (about 1.56 MiB, held on every GPU that loads the library until the
+ *   process exits); a call that would need more returns VP_ERR_STATIC_SCRATCH.  The call
+ *   allocates nothing itself (no cudaMalloc, cudaFree or allocating library routine).
+ *   Set-up: the first call on a device (or the first after a device reset) looks up the
+ *   buffer's device address with that device current.  CUDA loads a library's device code
+ *   lazily by default, so that first call is also when the runtime loads the router's kernels
+ *   and places the fixed buffer in device memory: make it before a host framework reserves
+ *   the GPU's memory for its own pool, and before any stream capture.
  *   All calls on a device share the buffer, which keeps the last call's contents; the parts
  *   that must start at zero are cleared at the start of every call.  Calls that overlap on
  *   the GPU (unordered streams or host threads) race on the buffer: serialise them.
- *   Device error bits (e.g. a NaN saliency) are cleared per call and not reported.
+ *   Device error bits (a wait that timed out, a NaN saliency) accumulate in the buffer's
+ *   error word until vp_router_noalloc_error reads them.
  */
 vp_status vp_router_noalloc(const vp_dims* dims, const vp_bf16* qkv, const vp_router_weights* rw,
                             const int32_t* force_modes, float* s, int32_t* modes, float* q_pool,
                             float* ctx, float* mean_v, float* r, void* stream);
+
+/* Reads and clears the device error word of vp_router_noalloc's fixed buffer on the current
+   device, as vp_read_device_error does for a workspace: enqueues a copy on `stream`,
+   synchronises that stream, writes the VP_DEVERR_* bits to *host_bits (host pointer).
+   Returns VP_ERR_DEVICE_TIMEOUT if the wait-timeout bit was set, else VP_OK.  Allocates
+   nothing. */
+vp_status vp_router_noalloc_error(uint32_t* host_bits, void* stream);
 
 /* Kernel classes reported by the launch profiler. */
 #define VP_KERNEL_GEMM 0

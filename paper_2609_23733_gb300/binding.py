@@ -80,6 +80,7 @@ _SIGS = [
     ("vp_router_noalloc", c_int32, [POINTER(VpDims), c_void_p, POINTER(VpRouterWeights), c_void_p,
                                     c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                     c_void_p]),
+    ("vp_router_noalloc_error", c_int32, [POINTER(c_uint32), c_void_p]),
     ("vp_bin_heads", c_int32, [c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                c_void_p]),
     ("vp_head_attention", c_int32, [POINTER(VpDims), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
@@ -266,6 +267,15 @@ def vp_router_noalloc(dm, qkv, rw: VpRouterWeights, force_modes, s, modes, q_poo
     _check(lib().vp_router_noalloc(ctypes.byref(dm), _p(qkv), ctypes.byref(rw), _p(force_modes), _p(s),
                                    _p(modes), _p(q_pool), _p(ctx), _p(mean_v), _p(r), _stream(stream)),
            "vp_router_noalloc")
+
+
+def vp_router_noalloc_error(stream=None) -> int:
+    """Reads and clears the device error bits of vp_router_noalloc's fixed buffer."""
+    bits = c_uint32(0)
+    st = lib().vp_router_noalloc_error(ctypes.byref(bits), _stream(stream))
+    if st not in (0, 5):
+        _check(st, "vp_router_noalloc_error")
+    return bits.value
 
 
 def vp_bin_heads(H, N, modes, head_ids, offsets, work=None, n_work=None, stream=None):

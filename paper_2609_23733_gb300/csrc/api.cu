@@ -119,17 +119,8 @@ cudaError_t make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t cols,
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-}  // namespace vp
-
-using namespace vp;
-
-namespace {
-
-constexpr size_t kAlign = 256;
-size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
-
-bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-
+// ------------------------------------------------------------------ shared argument checks
+// (also used by the fixed-scratch router, router_noalloc.cu)
 vp_status check_dims(const vp_dims* dm) {
   if (!dm) return VP_ERR_INVALID_ARG;
   if (dm->d != kHeadDim || dm->L != kHidden || dm->H < 1 || dm->H > kMaxHeads || dm->N < 1)
@@ -143,6 +134,43 @@ vp_status check_dims(const vp_dims* dm) {
     return VP_ERR_INVALID_ARG;  // those two modify the §4.3 surrogate, which linear attention replaces
   return VP_OK;
 }
+
+vp_status check_router_weights(const vp_router_weights* rw) {
+  if (!rw || !rw->W || !rw->U || !rw->w) return VP_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(rw->W) & 15u) || (reinterpret_cast<uintptr_t>(rw->U) & 15u))
+    return VP_ERR_ALIGNMENT;
+  return VP_OK;
+}
+
+RouterArgs make_router_args(const vp_dims* dm, const vp_bf16* qkv, const vp_router_weights* rw,
+                            const int32_t* force_modes) {
+  RouterArgs a{};
+  a.N = dm->N;
+  a.H = dm->H;
+  a.tau_low = dm->tau_low;
+  a.tau_high = dm->tau_high;
+  a.variant = dm->variant;
+  a.qkv = reinterpret_cast<const __nv_bfloat16*>(qkv);
+  a.W = reinterpret_cast<const __nv_bfloat16*>(rw->W);
+  a.U = reinterpret_cast<const __nv_bfloat16*>(rw->U);
+  a.w = reinterpret_cast<const __nv_bfloat16*>(rw->w);
+  a.bW = rw->bW;
+  a.bU = rw->bU;
+  a.beta = rw->beta;
+  a.force_modes = force_modes;
+  return a;
+}
+
+}  // namespace vp
+
+using namespace vp;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 vp_status check_device() {
   if (!device_is_sm103()) return VP_ERR_UNSUPPORTED_DEVICE;
@@ -256,12 +284,6 @@ vp_status from_cuda(cudaError_t e) { return e == cudaSuccess ? VP_OK : VP_ERR_CU
     if (_s != VP_OK) return _s;        \
   } while (0)
 
-vp_status check_router_weights(const vp_router_weights* rw) {
-  if (!rw || !rw->W || !rw->U || !rw->w) return VP_ERR_INVALID_ARG;
-  if (!aligned16(rw->W) || !aligned16(rw->U)) return VP_ERR_ALIGNMENT;
-  return VP_OK;
-}
-
 vp_status check_surrogate_weights(const vp_surrogate_weights* sw) {
   if (!sw || !sw->g1_w || !sw->g1_b || !sw->g2_w || !sw->g2_b || !sw->d1_w || !sw->d1_b ||
       !sw->d2_w || !sw->d2_b)
@@ -269,25 +291,6 @@ vp_status check_surrogate_weights(const vp_surrogate_weights* sw) {
   if (!aligned16(sw->g1_w) || !aligned16(sw->g2_w) || !aligned16(sw->d1_w) || !aligned16(sw->d2_w))
     return VP_ERR_ALIGNMENT;
   return VP_OK;
-}
-
-RouterArgs make_router_args(const vp_dims* dm, const vp_bf16* qkv, const vp_router_weights* rw,
-                            const int32_t* force_modes) {
-  RouterArgs a{};
-  a.N = dm->N;
-  a.H = dm->H;
-  a.tau_low = dm->tau_low;
-  a.tau_high = dm->tau_high;
-  a.variant = dm->variant;
-  a.qkv = reinterpret_cast<const __nv_bfloat16*>(qkv);
-  a.W = reinterpret_cast<const __nv_bfloat16*>(rw->W);
-  a.U = reinterpret_cast<const __nv_bfloat16*>(rw->U);
-  a.w = reinterpret_cast<const __nv_bfloat16*>(rw->w);
-  a.bW = rw->bW;
-  a.bU = rw->bU;
-  a.beta = rw->beta;
-  a.force_modes = force_modes;
-  return a;
 }
 
 SurrogateArgs make_surrogate_args(const vp_surrogate_weights* sw) {

@@ -53,8 +53,18 @@ constexpr size_t kFaCountWords = (size_t)kFaTailUnits * 4 * 4;
 // sum_j phi(k_j)[c] v_j[e], then z_h [64] = sum_j phi(k_j), fp32.
 constexpr int kLinState = 64 * 64 + 64;
 
-// Bytes of the router's scratch (what vp_router touches).
-size_t router_scratch_bytes(int H);
+// Bytes of the router's scratch (what vp_router touches): laid out for kMaxHeads heads
+// whatever H is (carve_router_scratch).
+constexpr size_t router_scratch_bytes(int /*H*/) {
+  return ((size_t)256                                           // error word
+          + 512                                                 // counters
+          + (size_t)kMaxHeads * kPoolSplitMax * kPoolPartial * 4
+          + (size_t)kMaxHeads * kKeySplitMax * kKeyPartial * 4
+          + (size_t)kMaxHeads * 64 * 4 * 3                      // q_pool, ctx, mean_v
+          + (size_t)kMaxHeads * 4 * 4                           // key_stats, s, modes
+          + 256                                                 // head_ids, offsets
+          + 4095) & ~(size_t)4095;
+}
 // Router scratch + linear-attention state: the workspace of the head modes.
 size_t heads_scratch_bytes(int H);
 RouterScratch carve_router_scratch(void* ws, int H);
@@ -82,6 +92,14 @@ struct RouterArgs {
 
 cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_sms,
                           cudaStream_t st);
+
+// Host-side argument checks shared by the router entry points (api.cu): dims (shape, taus,
+// variant bits), router weights (presence, 16-byte alignment of W and U), and the
+// RouterArgs of a call (outputs left NULL).
+vp_status check_dims(const vp_dims* dm);
+vp_status check_router_weights(const vp_router_weights* rw);
+RouterArgs make_router_args(const vp_dims* dm, const vp_bf16* qkv, const vp_router_weights* rw,
+                            const int32_t* force_modes);
 cudaError_t launch_bin_heads(int H, int N, const int32_t* modes, int32_t* head_ids,
                              int32_t* offsets, int32_t* work, int32_t* n_work, cudaStream_t st);
 

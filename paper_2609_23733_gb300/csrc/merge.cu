@@ -141,8 +141,11 @@ __device__ __forceinline__ Segment segment_at(long long u, long long u_end, int 
 
 // (score, column) as one 64-bit key that orders like the argmax: higher score first, then the
 // lower column.  Float bits made monotone: negative values inverted, positive ones offset.
+// -0 and +0 are the same score, so -0 is keyed as +0 (else +0 at a higher column would beat
+// an equal -0 and break the lowest-column rule).
 __device__ __forceinline__ unsigned long long match_key(float v, int col) {
-  const uint32_t b = __float_as_uint(v);
+  uint32_t b = __float_as_uint(v);
+  if (b == 0x80000000u) b = 0u;
   const uint32_t ord = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
   return ((unsigned long long)ord << 32) | (unsigned long long)(~(uint32_t)col);
 }

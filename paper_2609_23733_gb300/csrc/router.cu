@@ -585,18 +585,6 @@ cudaError_t launch_wait_selftest(unsigned int* err, unsigned long long limit_ns,
   return cudaGetLastError();
 }
 
-size_t router_scratch_bytes(int H) {
-  (void)H;
-  size_t b = 256;                                                    // error word
-  b += 512;                                                          // counters
-  b += (size_t)kMaxHeads * kPoolSplitMax * kPoolPartial * 4;
-  b += (size_t)kMaxHeads * kKeySplitMax * kKeyPartial * 4;
-  b += (size_t)kMaxHeads * 64 * 4 * 3;                               // q_pool, ctx, mean_v
-  b += (size_t)kMaxHeads * 4 * 4;                                    // key_stats, s, modes
-  b += 256;                                                          // head_ids, offsets
-  return (b + 4095) & ~(size_t)4095;
-}
-
 size_t heads_scratch_bytes(int H) {
   return router_scratch_bytes(H) + (size_t)kMaxHeads * kLinState * 4 +
          (kFaPartFloats + kFaStatsFloats + kFaCountWords) * 4;

@@ -80,9 +80,21 @@ def test_host_side_validation(vp):
     assert lib.vp_router(ctypes.byref(dm), A + 8, ctypes.byref(rw), None, A, A, None, None, None, None, A, 1 << 30, None) == 3
     assert lib.vp_router(ctypes.byref(dm), A, ctypes.byref(null_rw), None, A, A, None, None, None, None, A, 1 << 30, None) == 1
     assert lib.vp_router(ctypes.byref(dm), A, ctypes.byref(rw), None, A, A, None, None, None, None, A, 16, None) == 6
-    # vp_router_noalloc: more heads than its fixed buffer holds
-    assert lib.vp_router_noalloc(ctypes.byref(vp.dims(300, H=33)), A, ctypes.byref(rw), None, A, A,
-                                 None, None, None, None, None) == 8
+    # vp_router_noalloc: the checks of vp_router (H outside 1..32 is a shape error, as there;
+    # unknown or conflicting variant bits; missing outputs or weights; alignment)
+    na = lambda d, q=A, r=rw, s=A: lib.vp_router_noalloc(None if d is None else ctypes.byref(d), q,
+                                                         ctypes.byref(r), None, s, A, None, None, None,
+                                                         None, None)
+    assert na(None) == 1
+    assert na(vp.dims(300, H=33)) == 2
+    assert na(bad) == 2
+    assert na(vp.dims(300, variant=16)) == 1
+    assert na(vp.dims(300, variant=8 | 2)) == 1
+    assert na(dm, s=None) == 1
+    assert na(dm, r=null_rw) == 1
+    assert na(dm, q=A + 8) == 3
+    # its error reader needs somewhere to write the bits
+    assert lib.vp_router_noalloc_error(None, None) == 1
     # vp_linear: shapes and alignment
     assert lib.vp_linear(100, 12, 64, A, A, None, 0, None, None, A, None) == 2
     assert lib.vp_linear(100, 256, 60, A, A, None, 0, None, None, A, None) == 2
