@@ -17,11 +17,21 @@ def round_bf16(x) -> np.ndarray:
     bf16 keeps 8 significant bits (1 implicit + 7 stored) and float32's
     exponent range; below 2^-126 the spacing stays 2^-133 (subnormals).
     The result is returned as float64 (exactly representable).
+
+    In bf16's normal range the rounding is done on the float64 bit pattern: of the 52
+    stored mantissa bits, bf16 keeps the top 7, so the low 45 bits are dropped after
+    adding half of their weight (2^44), minus one unless the lowest kept bit is odd (ties
+    go to the even neighbour); a carry out of the mantissa moves to the next binade, as it
+    should.  Below 2^-126 the value is rounded at the fixed spacing 2^-133 instead.
     """
-    x = np.asarray(x, dtype=np.float64)
-    _, e = np.frexp(x)                     # x = m * 2^e, 0.5 <= |m| < 1
-    shift = np.maximum(e - 8, -133)        # spacing of bf16 values near x
-    y = np.ldexp(np.rint(np.ldexp(x, -shift)), shift)   # rint: half to even
+    x = np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+    b = x.view(np.uint64)
+    keep = (b >> np.uint64(45)) & np.uint64(1)
+    y = ((b + (np.uint64((1 << 44) - 1) + keep)) >> np.uint64(45) << np.uint64(45)).view(np.float64)
+    small = np.abs(x) < 2.0 ** -126
+    if np.any(small):  # bf16 subnormals: multiples of 2^-133 (rint: half to even)
+        y = np.where(small, np.ldexp(np.rint(np.ldexp(x, 133)), -133), y)
+    y = np.where(np.isfinite(x), y, x)
     over = np.abs(y) > BF16_MAX
     if np.any(over):
         y = np.where(over, np.copysign(np.inf, x), y)
