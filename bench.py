@@ -15,7 +15,8 @@ the dominant kernel class, timed with CUDA events recorded by the library around
 its launches inside the timed region.  ``cpu_baseline`` times the float64 oracle on a
 bounded sample of the same workload (rank 0, one GPU only).
 
---impl reference runs that oracle as the reference arm instead.
+--impl reference runs that oracle as the reference arm instead: each of its steps is the
+bounded CPU sample, scaled to a whole forward (an extrapolation, labelled as such).
 """
 from __future__ import annotations
 
@@ -185,6 +186,15 @@ def cpu_cores():
 
 
 # ------------------------------------------------------------------ arms
+def workload_config(world):
+    """The workload both arms report (the same dict, so that their lines compare)."""
+    return {"workload": WORKLOAD.name, "views": WORKLOAD.views, "image_px": WORKLOAD.image_px,
+            "tokens": WORKLOAD.N, "layers": WORKLOAD.layers, "dim": D, "heads": H, "head_dim": d,
+            "routing": "paper_mix (30 full / 162 surrogate / 192 mean of 384 heads)",
+            "parallelism": f"replicas{world}",
+            "l2": "inputs larger than L2 (281 MB tokens, 1.4 GB workspace)"}
+
+
 def run_reference(args):
     """The oracle as the reference arm: each step is the bounded CPU sample."""
     rank = int(os.environ.get("RANK", "0"))
@@ -194,21 +204,26 @@ def run_reference(args):
     routes = synth.paper_mix_modes(WORKLOAD.layers)
     w0 = synth.make_stack_weights(WORKLOAD.seed, 1)[0]
     x_bits = synth.make_tokens(WORKLOAD.seed, N)
-    times = []
+    times, walls = [], []
     desc = ""
     for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
         ms, desc, _ = oracle_sample(N, routes, w0, x_bits)
         if i >= args.warmup:
             times.append(ms)
+            walls.append(time.perf_counter() - t0)
     ms = float(np.median(times))
+    sample_s = float(np.median(walls))  # CPU time actually spent per step (the sample)
     value = WORKLOAD.views / (ms / 1e3)
-    cb = {"value": value, "unit": "views/s", "cores": cpu_cores(), "kind": "oracle", "sample": desc}
+    cb = {"value": value, "unit": "views/s", "cores": cpu_cores(), "kind": "oracle", "sample": desc,
+          "extrapolated": True, "sample_s_per_step": sample_s}
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "views/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD.name, "views": WORKLOAD.views, "tokens": N, "layers": WORKLOAD.layers,
-                   "routing": "paper_mix"},
+        "config": workload_config(args.gpus),
+        "extrapolated": True,
+        "sample_s_per_step": sample_s,
         "cpu_baseline": cb,
         "e2e": {"value": value, "unit": "views/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
 
@@ -348,18 +363,17 @@ def run_ours(args):
 
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
+        t0 = time.perf_counter()
         ms_cpu, desc, _ = oracle_sample(N, routes, host_w[0], x_bits)
         cpu = {"value": WORKLOAD.views / (ms_cpu / 1e3), "unit": "views/s", "cores": cpu_cores(),
-               "kind": "oracle", "sample": desc}
+               "kind": "oracle", "sample": desc, "extrapolated": True,
+               "sample_s": time.perf_counter() - t0}
 
     line = {
         "metric": METRIC, "value": value, "unit": "views/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": WORKLOAD.name, "views": WORKLOAD.views, "image_px": WORKLOAD.image_px,
-                   "tokens": N, "layers": L, "dim": D, "heads": H, "head_dim": d,
-                   "routing": "paper_mix (30 full / 162 surrogate / 192 mean of 384 heads)",
-                   "parallelism": f"replicas{world}", "l2": "inputs larger than L2 (281 MB tokens, 1.4 GB workspace)"},
+        "config": workload_config(world),
         "e2e": {"value": job_value(e2e_ms, world, WORKLOAD.views), "unit": "views/s",
                 "h2d_bytes_per_step": int(x_host.numel() * 2), "d2h_bytes_per_step": int(y_host[0].numel() * 2),
                 "ms_per_step": e2e_ms, "steps": e2e_steps,
@@ -388,6 +402,8 @@ def run_ours(args):
         line["token_merging_s100"] = tome_probe(vpb, dev, N, dws, fm)
     if args.mix:
         line["mix_sweep_s64"] = mix_probe(vpb, dev, pk)
+    if args.saliency:
+        line["saliency_router_vs_exact"] = saliency_probe(vpb, dev)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
@@ -588,6 +604,86 @@ def mix_probe(vpb, dev, pk, steps=3, warmup=2):
             "speedup_vs_all_full": {f"{r['full_fraction']:.2f}": t[-1] / r["ms_per_layer"] for r in rows}}
 
 
+# ------------------------------------------------------------------ router vs exact saliency
+def rank_correlation(a, b):
+    """Spearman's rank correlation of two samples (average ranks for ties)."""
+    def ranks(v):
+        v = np.asarray(v, np.float64)
+        order = np.argsort(v, kind="stable")
+        r = np.empty(len(v))
+        r[order] = np.arange(len(v), dtype=np.float64)
+        for u in np.unique(v):  # ties share their average rank
+            m = v == u
+            r[m] = r[m].mean()
+        return r
+    ra, rb = ranks(a), ranks(b)
+    ra -= ra.mean()
+    rb -= rb.mean()
+    den = np.sqrt((ra * ra).sum() * (rb * rb).sum())
+    return float((ra * rb).sum() / den) if den > 0 else float("nan")
+
+
+def route_of(s, tau_low=0.01, tau_high=0.2):
+    """§4.2 routing equation applied to a saliency (float32 comparisons; NaN -> full)."""
+    s = np.float32(s)
+    if np.isnan(s) or s >= np.float32(tau_high):
+        return synth.MODE_FULL
+    return synth.MODE_MEAN if s <= np.float32(tau_low) else synth.MODE_SURROGATE
+
+
+def saliency_agreement(s_router, s_exact):
+    """How the router's saliency s_h (§4.1) ranks and routes the heads against the exact
+    MaxAttn saliency s_h^attn = max_ij A_h[i, j] (§3, the quantity the router is distilled to
+    approximate): per-head pairs, Spearman's rank correlation, and the 3 x 3 table of routes
+    (rows: route under s_h; columns: route under s_h^attn; order mean, surrogate, full)."""
+    r_router = [route_of(v) for v in s_router]
+    r_exact = [route_of(v) for v in s_exact]
+    table = np.zeros((3, 3), np.int64)
+    for a, b in zip(r_router, r_exact):
+        table[a, b] += 1
+    return {"pairs": [[float(a), float(b)] for a, b in zip(s_router, s_exact)],
+            "spearman": rank_correlation(s_router, s_exact),
+            "routes_router": r_router, "routes_exact": r_exact,
+            "route_table": table.tolist(), "routes_agree": int(np.trace(table))}
+
+
+def saliency_probe(vpb, dev):
+    """Router vs exact saliency on one S=8 and one S=64 layer (518 px): every head forced to
+    full mode, so the attention kernel's epilogue returns the exact s_h^attn of all 16 heads
+    beside the router's s_h.  The routers are untrained (Xavier weights); their temperatures
+    beta_h are spread geometrically over [1, 3000] so that the router's saliencies cover all
+    three bands of §4.2.  An untrained router has no reason to track s_h^attn: the report is
+    the measurement, not a claim of agreement."""
+    import torch
+    out = {}
+    for key in ("s8_layer_biased", "s64_mix_sweep"):
+        wl = synth.WORKLOADS[key]
+        N = wl.N
+        w = synth.make_layer_weights(synth.rng(wl.seed + 500))
+        w["r_beta"] = np.geomspace(1.0, 3000.0, H).astype(np.float32)
+        dw = vpb.to_device(w, dev)
+        x = vpb.bf16_from_bits(synth.make_tokens(wl.seed, N), dev)
+        dm = vpb.dims(N, H)
+        ws = vpb.workspace(dm, vpb.VP_WS_LAYER, dev)
+        y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
+        s = torch.zeros(H, device=dev)
+        s_attn = torch.zeros(H, device=dev)
+        modes = torch.zeros(H, dtype=torch.int32, device=dev)
+        fm = torch.full((H,), synth.MODE_FULL, dtype=torch.int32, device=dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        vpb.vp_moh_global_attention(dm, x, dw["w_qkv"], dw["b_qkv"], dw["w_o"], dw["b_o"],
+                                    vpb.router_weights(dw), vpb.surrogate_weights(dw), fm, y, None, None,
+                                    s, modes, ws, s_attn_out=s_attn)
+        b.record()
+        torch.cuda.synchronize()
+        rep = saliency_agreement(s.cpu().numpy(), s_attn.cpu().numpy())
+        rep.update({"workload": wl.name, "views": wl.views, "tokens": N, "ms_layer_all_full": a.elapsed_time(b),
+                    "router_beta": "geomspace(1, 3000, 16)"})
+        out[key] = rep
+    return out
+
+
 def full_attention_probe(vpb, dev, N, dw, pk):
     """All 16 heads in full mode over N tokens (the forced all-full layer of the target)."""
     import torch
@@ -746,6 +842,8 @@ def main():
     ap.add_argument("--no-qk", dest="qk", action="store_false")
     ap.add_argument("--no-tome", dest="tome", action="store_false")
     ap.add_argument("--no-mix", dest="mix", action="store_false", help="skip the S=64 routing-mix sweep")
+    ap.add_argument("--no-saliency", dest="saliency", action="store_false",
+                    help="skip the router-vs-exact saliency report")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
                                               "surrogate", "mean", "bin", "merge"],
                     default=None,
