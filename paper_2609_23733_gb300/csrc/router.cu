@@ -491,8 +491,10 @@ __global__ void __launch_bounds__(kKeyThreads) router_keys_kernel(RouterArgs a, 
     if (a.ctx_out) a.ctx_out[h * 64 + tid] = ctx;
     if (a.mean_v_out) a.mean_v_out[h * 64 + tid] = mv;
     if (tid == 0) {
-      // s_h = max_j r_h(j) = 2^(max - max) / sum_j 2^(l_j - max).
-      const float s = 1.f / ll;
+      // s_h = max_j r_h(j) = 2^(max - max) / sum_j 2^(l_j - max).  No finite logit at all
+      // (a NaN pooled query makes every logit NaN, and NaN never raises the running maximum)
+      // means r_h is NaN, and so is s_h.
+      const float s = Mx == -INFINITY ? __int_as_float(0x7fc00000) : 1.f / ll;
       bool nan;
       int mode = select_mode(s, a.tau_low, a.tau_high, nan);
       if (nan) atomicOr(sc.err, VP_DEVERR_NAN_SALIENCY);

@@ -121,6 +121,7 @@ def _s32_oracle():
     return {"wl": wl, "wts": wts, "x_bits": x_bits, "inputs": inputs, "infos": infos, "out": X}
 
 
+@pytest.mark.slow
 @pytest.mark.parametrize("blk", [0, 11, 23])
 def test_stack_s32_block_against_oracle(blk, _s32_oracle):
     """Full size S=32 (43,968 tokens): blocks 0, 11 and 23 of the 24-block stack, each run on
@@ -135,6 +136,7 @@ def test_stack_s32_block_against_oracle(blk, _s32_oracle):
     compare(got, oracle.bf16_bits_to_f64(want), rel=BF16_STEP, what=f"S=32 block {blk}")
 
 
+@pytest.mark.slow
 def test_stack_s32_24_blocks_against_oracle(_s32_oracle):
     """The whole S=32 stack, 24 blocks on the GPU from the tokens, against the oracle's 24
     blocks: routes of every block exact, the output within the depth budget of
