@@ -16,8 +16,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libvp.so")
-SOURCES = ["api.cu", "router.cu", "attn_full.cu", "heads_cheap.cu", "gemm.cu", "layernorm.cu",
-           "router_noalloc.cu", "merge.cu"]
+SOURCES = ["api.cu", "router.cu", "attn_full.cu", "heads_cheap.cu", "heads_cheap_tc.cu", "gemm.cu",
+           "layernorm.cu", "router_noalloc.cu", "merge.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

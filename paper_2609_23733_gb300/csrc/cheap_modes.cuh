@@ -103,7 +103,7 @@ __device__ __forceinline__ void linear_stage(const HeadAttnArgs& a, LinSmem& sm,
 // phi(Q) rounded to bf16, S_h as hi + lo bf16 parts, fp32 accumulation) with the same
 // permuted reduction index as surrogate_rows; the denominator in fp32 from the same rows.
 // Not inlined: its registers then do not add to those of the kernel's other paths.
-__device__ __noinline__ void linear_rows(const HeadAttnArgs& a, const LinSmem& sm, int h,
+static __device__ __noinline__ void linear_rows(const HeadAttnArgs& a, const LinSmem& sm, int h,
                                             int chunk, int w, int lane) {
   const int N = a.N, H = a.H;
   const size_t row_pitch = (size_t)3 * H * kHeadDim;

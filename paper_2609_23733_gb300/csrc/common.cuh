@@ -248,6 +248,18 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
       : "r"(taddr));
 }
 
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+  uint32_t* r = reinterpret_cast<uint32_t*>(v);
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
   const uint32_t* r = reinterpret_cast<const uint32_t*>(v);
   asm volatile(
@@ -270,6 +282,14 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
       "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
       "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
       "r"(r[15])
+      : "memory");
+}
+
+// 8 consecutive 32-bit columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
       : "memory");
 }
 
@@ -348,11 +368,11 @@ __device__ __forceinline__ float gelu_as(float x) {
   return 0.5f * x * (1.f + erf_as(x * 0.70710678118654752f));
 }
 
-// The same GELU for two values with packed f32x2 arithmetic.  With z = x / sqrt 2 and
+// Twice the same GELU for two values with packed f32x2 arithmetic.  With z = x / sqrt 2 and
 // erf(z) = sign(z) (1 - poly(t) e^{-z^2}) from 7.1.26, x (1 + erf(z)) = x + |x| r with
-// r = 1 - poly(t) e^{-z^2}, so no sign transfer is needed: gelu = 0.5 (x + |x| r).  The
+// r = 1 - poly(t) e^{-z^2}, so no sign transfer is needed: 2 gelu = x + |x| r.  The
 // polynomial is evaluated with negated coefficients, so that r = 1 + poly'(t) e^{-z^2}.
-__device__ __forceinline__ float2 gelu_as2(float2 x) {
+__device__ __forceinline__ float2 gelu2_as2(float2 x) {
   const float kP = 0.3275911f * 0.70710678118654752f;  // p / sqrt 2: t = 1 / (1 + p |z|)
   const float kE = -0.5f * 1.4426950408889634f;        // e^{-z^2} = 2^{kE x^2}
   const float2 ax = make_float2(fabsf(x.x), fabsf(x.y));
@@ -369,7 +389,12 @@ __device__ __forceinline__ float2 gelu_as2(float2 x) {
   const float2 q = fmul2(ax, fmul2(ax, make_float2(kE, kE)));
   const float2 e = make_float2(fast_exp2(q.x), fast_exp2(q.y));
   const float2 r = ffma2(p, e, make_float2(1.f, 1.f));
-  return fmul2(ffma2(ax, r, x), make_float2(0.5f, 0.5f));
+  return ffma2(ax, r, x);
+}
+
+// GELU of two values: half of gelu2_as2.
+__device__ __forceinline__ float2 gelu_as2(float2 x) {
+  return fmul2(gelu2_as2(x), make_float2(0.5f, 0.5f));
 }
 
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }

@@ -175,6 +175,13 @@ cudaError_t launch_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
   prof_before(VP_KERNEL_ATTN_FULL, st);  // both kernels: no event may separate them
   e = launch_full_heads(a, num_sms, st);
   if (e != cudaSuccess) return e;
+  if (!(a.variant & (VP_VARIANT_NO_RESIDUAL | VP_VARIANT_LINEAR_ATTENTION))) {
+    e = launch_cheap_heads_tc(a, num_sms, st);
+    prof_extra_launch();
+    prof_after(st);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(3 * num_sms);
   cfg.blockDim = dim3(kThreads);

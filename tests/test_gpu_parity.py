@@ -261,6 +261,36 @@ def test_head_modes_match_oracle(N):
     _check_saliency(s_attn, qkv, modes, f"N={N}")
 
 
+@pytest.mark.parametrize("N,modes", [(9999, [1] * 16), (4000, [1, 0] * 8), (300, [0, 1, 1, 0, 1, 1, 1, 0])])
+def test_surrogate_and_mean_heads_many_items(N, modes):
+    """Surrogate and mean heads over many 128-token items: every CTA takes items of several
+    heads in turn, so the surrogate weights of a head are loaded into a shared-memory slot
+    while the previous head's tiles still run; a ragged last item.  Every row against the
+    oracle (the oracle's own router supplies r_h and C_h)."""
+    H = len(modes)
+    modes = np.array(modes, np.int32)
+    g = synth.rng(N + H)
+    w = synth.make_layer_weights(g, D=H * 64, H=H, bias_std=0.1)
+    qkv_bits = synth.f32_to_bf16_bits(g.standard_normal((N, 3, H, 64)).astype(np.float32) * 1.5)
+    lw = oracle.load_layer(w)
+    qkv = oracle.bf16_bits_to_f64(qkv_bits).reshape(N, 3, H, 64)
+    ctx, mean_v = np.zeros((H, 64)), np.zeros((H, 64))
+    want = np.zeros((N, H, 64))
+    for h in range(H):
+        Q, K, V = qkv[:, 0, h], qkv[:, 1, h], qkv[:, 2, h]
+        _, _, r, _ = oracle.layer.head_router(Q, K, lw, h)
+        ctx[h], mean_v[h] = r @ V, V.mean(0)
+        if modes[h] == 1:
+            mg = (lw["s_g1_w"][h], lw["s_g1_b"][h], lw["s_g2_w"][h], lw["s_g2_b"][h])
+            md = (lw["s_d1_w"][h], lw["s_d1_b"][h], lw["s_d2_w"][h], lw["s_d2_b"][h])
+            want[:, h], _ = oracle.surrogate_attention(V, r, mg, md)
+        else:
+            want[:, h], _ = oracle.mean_pooling(V)
+    got = _run_heads(qkv_bits, w, N, H, modes, ctx, mean_v)
+    for h in range(H):
+        compare(got[:, h], oracle.round_bf16(want[:, h]), what=f"N={N} head {h} mode {modes[h]}")
+
+
 @pytest.mark.parametrize("N", [5000, 9999])
 def test_full_attention_many_items(N):
     # More (head, query pair) work items than CTAs: every CTA runs several items in turn and
