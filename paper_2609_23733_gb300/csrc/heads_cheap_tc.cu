@@ -26,13 +26,15 @@
 //              head before the previous one have completed);
 //   warp 1     TMEM owner (512 columns) and MMA issue: the first layer of the next tile and
 //              the second layer of a tile whose H is written, each as soon as it is ready;
-//   warps 2-9, 10-17  two epilogue groups of eight warps, each with 256 TMEM columns; group g
-//              takes tiles t = g (mod 2).  Its j-th tile keeps D1, then D2g | D2d, in the
+//   warps 2-9, 10-17  two epilogue groups of eight warps, each with 256 TMEM columns; group
+//              g takes tiles t = g (mod 2).  Its j-th tile keeps D1, then D2g | D2d, in the
 //              128-column half j & 1 and H in the first 64 columns of the other half, so the
-//              first layer of its next tile (the other half) runs while it reads D2.
-//              The two warps of a TMEM lane quarter split a token row's columns: half 0 the
-//              gamma hidden units and output columns 0..31, half 1 the delta hidden units and
-//              output columns 32..63.
+//              first layer of its next tile (the other half) runs while it reads D2.  The
+//              two warps of a TMEM lane quarter split a token row's columns (kTcParts).
+// The register file is split between the four SM sub-partitions: 18 warps put 5 on some of
+// them, which caps a thread at 96 registers (16,384 / (5 x 32), in steps of 8).  Three warps
+// per lane quarter (26 warps, 72 registers) measured slower: 0.301 vs 0.269 ms for 16 heads
+// at 137,400 tokens.
 // Every wait is bounded (mbar_wait); on timeout the CTA records VP_DEVERR_WAIT_TIMEOUT, stops,
 // waits (bounded) for its own copies and MMAs, frees TMEM and exits.  The groups agree on
 // stopping through reduction barriers, so that no thread is left at a named barrier.
@@ -48,7 +50,16 @@ constexpr int kTcTile = 128;      // tokens per item
 constexpr int kTcStages = 4;      // V tiles in flight
 constexpr int kTcGroups = 2;      // epilogue groups (= TMEM accumulators)
 constexpr int kTcBatch = 4;       // items taken from the counter at a time
-constexpr int kTcThreads = 64 + 256 * kTcGroups;
+constexpr int kTcParts = 2;       // epilogue warps per TMEM lane quarter in a group
+constexpr int kGroupThreads = 128 * kTcParts;
+constexpr int kTcThreads = 64 + kGroupThreads * kTcGroups;
+// A row's work split over the kTcParts warps of its lane quarter: part p takes the chunk
+// range [begin(p), begin(p + 1)) of the n chunks, as even as possible.  The first layer's
+// 8 chunks go in part order and the second layer's 4 in reverse, so that a part short of
+// first-layer chunks takes more second-layer ones.
+__host__ __device__ constexpr int part_begin(int p, int n) { return (p * n + kTcParts - 1) / kTcParts; }
+constexpr int kMaxGChunks = (8 + kTcParts - 1) / kTcParts;
+constexpr int kMaxFChunks = (4 + kTcParts - 1) / kTcParts;
 constexpr uint32_t kTcTmemCols = 512;
 constexpr uint32_t kVTileBytes = kTcTile * 64 * 2;
 constexpr uint32_t kW1Bytes = 128 * 64 * 2;  // [W1v_gamma; W1v_delta]: 128 hidden x 64 inputs
@@ -76,17 +87,17 @@ struct TcSmem {
   int abort_flag;
 };
 
-// Barrier over the 256 threads of an epilogue group (named barrier 1 + g) that also returns
+// Barrier over the threads of an epilogue group (named barrier 1 + g) that also returns
 // whether p held on every one of them.
 __device__ __forceinline__ bool group_all(bool p, int g) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
       "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.and.pred po, %2, 256, pi;\n\t"
+      "bar.red.and.pred po, %2, %3, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
-      : "r"((uint32_t)p), "r"(1 + g)
+      : "r"((uint32_t)p), "r"(1 + g), "n"(kGroupThreads)
       : "memory");
   return r != 0;
 }
@@ -121,7 +132,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
     }
     for (int g = 0; g < kTcGroups; ++g) {
       mbar_init(&sm.d1_full[g], 2);  // the MMA commit (or a stand-in) + the item hand-over
-      mbar_init(&sm.h_full[g], 256);
+      mbar_init(&sm.h_full[g], kGroupThreads);
       mbar_init(&sm.d2_full[g], 1);
       mbar_init(&sm.taken[g], 1);      // the group has read a tile's item and left its last one
     }
@@ -424,12 +435,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
   } else {
     // ------------------------------------------------------------ epilogue groups
     const int e = warp - 2;
-    const int g = e >> 3, half = (e >> 2) & 1;
-    const int gt = tid - 64 - 256 * g;       // 0..255 within the group
-    const int quarter = warp & 3;            // TMEM lanes this warp may access
-    const int row = quarter * 32 + lane;     // token row of the tile = TMEM lane
+    const int g = e / (4 * kTcParts), part = (e % (4 * kTcParts)) >> 2;
+    const int gt = tid - 64 - kGroupThreads * g;  // 0 .. kGroupThreads - 1 within the group
+    const int quarter = warp & 3;                 // TMEM lanes this warp may access
+    const int row = quarter * 32 + lane;          // token row of the tile = TMEM lane
     const uint32_t t_grp = tmem + ((uint32_t)(quarter * 32) << 16) + g * 256;
     unsigned char* yrow = reinterpret_cast<unsigned char*>(sm.ys[g]) + row * 128;
+    // This warp's share of a row: hidden-unit chunks [g0, g1) of 16 (first layer, H) and
+    // output-column chunks [f0, f1) of 16 (second layer, y).
+    const int g0 = part_begin(part, 8), g1 = part_begin(part + 1, 8);
+    const int f0 = part_begin(kTcParts - 1 - part, 4), f1 = part_begin(kTcParts - part, 4);
     uint32_t sj = 0;  // surrogate tiles of this group
     bool ok = true;
     for (uint32_t j = 0;; ++j) {
@@ -451,24 +466,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
       const uint32_t t_h = t_grp + ((j & 1) ^ 1) * 128;
       if (surr) {
         // H = 2 GELU(D1 + c1) as bf16 pairs (the factor 2 is exact in bf16 and is taken out
-        // of the second layer's results): this half's 64 hidden units (D1 columns 64 half ..
-        // +64) into H columns 32 half .. +32.  Each chunk's TMEM load is in flight while the
-        // chunk before it is computed.
-        const int u0 = 64 * half;
+        // of the second layer's results): chunk c of 16 hidden units (D1 columns 16 c ..)
+        // into H columns 8 c .. + 8.  Each chunk's TMEM load is in flight while the chunk
+        // before it is computed.
         float vb[2][16];
-        tmem_ld16(t_acc + u0, vb[0]);
+        tmem_ld16(t_acc + 16 * g0, vb[0]);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {  // chunk c: units u0 + 16 c .. +16; the next one loads meanwhile
+        for (int i = 0; i < kMaxGChunks; ++i) {
+          const int c = g0 + i;
+          if (c >= g1) break;
           tmem_wait_ld();
-          if (c < 3) tmem_ld16(t_acc + u0 + 16 * (c + 1), vb[(c + 1) & 1]);
+          if (c + 1 < g1) tmem_ld16(t_acc + 16 * (c + 1), vb[(i + 1) & 1]);
           uint32_t hw[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const float2 cc = *reinterpret_cast<const float2*>(&c1[u0 + 16 * c + 2 * i]);
-            const float2 x = gelu2_as2(fadd2(make_float2(vb[c & 1][2 * i], vb[c & 1][2 * i + 1]), cc));
-            hw[i] = pack_bf16x2(x.x, x.y);
+          for (int q = 0; q < 8; ++q) {
+            const float2 cc = *reinterpret_cast<const float2*>(&c1[16 * c + 2 * q]);
+            const float2 x = gelu2_as2(fadd2(make_float2(vb[i & 1][2 * q], vb[i & 1][2 * q + 1]), cc));
+            hw[q] = pack_bf16x2(x.x, x.y);
           }
-          tmem_st8(t_h + u0 / 2 + 8 * c, hw);
+          tmem_st8(t_h + 8 * c, hw);
         }
         tmem_wait_st();
         tc_fence_before();
@@ -482,44 +498,47 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
       if (!ok) break;
       if (gt == 0) mbar_arrive(&sm.taken[g]);  // every thread has read this tile's item
       if (surr) {
-        // y = C + sigma(D2g + b2g) (.) (D2d + b2d) for this half's 32 output columns, from
+        // y = C + sigma(D2g + b2g) (.) (D2d + b2d) for chunk c of 16 output columns, from
         // D2' = 2 D2: sigma(u) = 1 / (1 + 2^(-log2(e) u)) with the exponent
         // -log2(e) / 2 D2g' + nbg, nbg = -log2(e) b2g held per head.
         tc_fence_after();
-        const int c0 = 32 * half;
-        float og[32], od[32];
-        tmem_ld32(t_acc + c0, og);
-        tmem_ld32(t_acc + 64 + c0, od);
-        tmem_wait_ld();
         const float kS = -0.5f * 1.4426950408889634f;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {  // 16-byte chunk jc of the row sits at chunk jc ^ (row & 7)
-          uint32_t yw[4];
+        for (int i = 0; i < kMaxFChunks; ++i) {
+          const int c = f0 + i;
+          if (c >= f1) break;
+          float og[16], od[16];
+          tmem_ld16(t_acc + 16 * c, og);
+          tmem_ld16(t_acc + 64 + 16 * c, od);
+          tmem_wait_ld();
+          uint32_t yw[8];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int k = 4 * q + i, col = c0 + 2 * k;
+          for (int q = 0; q < 8; ++q) {
+            const int col = 16 * c + 2 * q;
             const float2 C = *reinterpret_cast<const float2*>(&cx[col]);
             const float2 nbg = *reinterpret_cast<const float2*>(&b2[col]);
             const float2 bd = *reinterpret_cast<const float2*>(&b2[64 + col]);
-            const float2 ea = ffma2(make_float2(og[2 * k], og[2 * k + 1]), make_float2(kS, kS), nbg);
+            const float2 ea = ffma2(make_float2(og[2 * q], og[2 * q + 1]), make_float2(kS, kS), nbg);
             const float2 den = fadd2(make_float2(fast_exp2(ea.x), fast_exp2(ea.y)), make_float2(1.f, 1.f));
             float2 sg;
             asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(sg.x) : "f"(den.x));
             asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(sg.y) : "f"(den.y));
-            const float2 dl = ffma2(make_float2(od[2 * k], od[2 * k + 1]), make_float2(0.5f, 0.5f), bd);
+            const float2 dl = ffma2(make_float2(od[2 * q], od[2 * q + 1]), make_float2(0.5f, 0.5f), bd);
             const float2 y2 = ffma2(sg, dl, C);
-            yw[i] = pack_bf16x2(y2.x, y2.y);
+            yw[q] = pack_bf16x2(y2.x, y2.y);
           }
-          const int jc = c0 / 8 + q;
-          *reinterpret_cast<uint4*>(yrow + ((jc ^ (row & 7)) << 4)) = make_uint4(yw[0], yw[1], yw[2], yw[3]);
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {  // 16-byte chunk jc of the row sits at chunk jc ^ (row & 7)
+            const int jc = 2 * c + q;
+            *reinterpret_cast<uint4*>(yrow + ((jc ^ (row & 7)) << 4)) =
+                make_uint4(yw[4 * q], yw[4 * q + 1], yw[4 * q + 2], yw[4 * q + 3]);
+          }
         }
         tc_fence_before();
-      } else {  // Broadcast(mean of V_h): this half's 32 columns
-        const float4* m = reinterpret_cast<const float4*>(a.mean_v + h * 64 + 32 * half);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int jc = 4 * half + q;
-          const float4 m0 = __ldg(m + 2 * q), m1 = __ldg(m + 2 * q + 1);
+      } else {  // Broadcast(mean of V_h): this warp's output-column chunks
+        const float4* m = reinterpret_cast<const float4*>(a.mean_v + h * 64);
+        for (int jc = 2 * f0; jc < 2 * f1; ++jc) {
+          const float4 m0 = __ldg(m + 2 * jc), m1 = __ldg(m + 2 * jc + 1);
           *reinterpret_cast<uint4*>(yrow + ((jc ^ (row & 7)) << 4)) =
               make_uint4(pack_bf16x2(m0.x, m0.y), pack_bf16x2(m0.z, m0.w), pack_bf16x2(m1.x, m1.y),
                          pack_bf16x2(m1.z, m1.w));
