@@ -24,13 +24,21 @@ namespace {
 
 constexpr int kKeyThreads = 256;
 
-// tanh(x) * sigma(y) for the pooling logits of §4.1, two at a time on packed f32x2 pairs, in a
-// form that needs no clamps:
-// tanh(x) = sign(x) (1 - e^{-2|x|}) / (1 + e^{-2|x|}) with e^{-2|x|} <= 1, and
-// sigma(y) = 1 / (1 + e^{-y}), whose e^{-y} may overflow to +inf, giving 0 as it should.
+// max(a, b) that returns NaN when either is NaN (fmaxf would return the other operand).
+__device__ __forceinline__ float max_nan(float a, float b) {
+  float d;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+  return d;
+}
+
+// tanh(x) * sigma(y) for the pooling logits of §4.1, two at a time on packed f32x2 pairs:
+// tanh(x) sigma(y) = (1 - E) / ((1 + E)(1 + F)) with E = e^{-2x}, F = e^{-y}.  x is floored at
+// -40 so that E stays finite (tanh(-40) is -1 in float); a huge F (y << 0) makes the
+// denominator infinite and the product 0, as sigma(y) -> 0 requires.  NaNs propagate.
 __device__ __forceinline__ float2 tanh_times_sigmoid2(float2 x, float2 y) {
   const float kLog2e = 1.4426950408889634f;
-  const float2 a = fmul2(make_float2(fabsf(x.x), fabsf(x.y)), make_float2(-2.f * kLog2e, -2.f * kLog2e));
+  const float2 xc = make_float2(max_nan(x.x, -40.f), max_nan(x.y, -40.f));
+  const float2 a = fmul2(xc, make_float2(-2.f * kLog2e, -2.f * kLog2e));
   const float2 b = fmul2(y, make_float2(-kLog2e, -kLog2e));
   const float2 ea = make_float2(fast_exp2(a.x), fast_exp2(a.y));
   const float2 eb = make_float2(fast_exp2(b.x), fast_exp2(b.y));
@@ -39,8 +47,7 @@ __device__ __forceinline__ float2 tanh_times_sigmoid2(float2 x, float2 y) {
   float2 r;
   asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r.x) : "f"(den.x));
   asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r.y) : "f"(den.y));
-  const float2 t = fmul2(num, r);
-  return make_float2(copysignf(t.x, x.x), copysignf(t.y, x.y));
+  return fmul2(num, r);
 }
 
 __device__ __forceinline__ void token_range(int N, int n_split, int split, int align, int& t0,
@@ -111,7 +118,10 @@ struct PoolTcSmem {
   int abort_flag;
 };
 
-__global__ void __launch_bounds__(kPoolTcThreads)
+// kBias: the optional biases inside tanh and sigma (bW, bU) are given; without them (the
+// paper's form) their adds and loads are left out of the per-unit loop.
+template <bool kBias>
+__global__ void __launch_bounds__(kPoolTcThreads, 2)  // two CTAs per SM (TMEM: 2 x 256 columns)
     router_pool_tc_kernel(const __grid_constant__ CUtensorMap tmap_q,
                           const __grid_constant__ CUtensorMap tmap_w,
                           const __grid_constant__ CUtensorMap tmap_u, RouterArgs a,
@@ -234,25 +244,27 @@ __global__ void __launch_bounds__(kPoolTcThreads)
       tc_fence_after();
       float e2x = 0.f, e2y = 0.f;
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float zw[32], zu[32];
-        tmem_ld32(t_lane + ab * 128 + 32 * half, zw);
-        tmem_ld32(t_lane + ab * 128 + 64 + 32 * half, zu);
+      for (int qtr = 0; qtr < 4; ++qtr) {  // 16 + 16 accumulator columns at a time
+        float zw[16], zu[16];
+        tmem_ld16(t_lane + ab * 128 + 16 * qtr, zw);
+        tmem_ld16(t_lane + ab * 128 + 64 + 16 * qtr, zu);
         tmem_wait_ld();
-        if (half == 1) {  // the accumulator is in registers: back to the MMA warp
+        if (qtr == 3) {  // the accumulator is in registers: back to the MMA warp
           tc_fence_before();
           mbar_arrive(&sm.acc_empty[ab]);
         }
         float2 pe = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const int l = 32 * half + 2 * k;
-          const float2 bw = *reinterpret_cast<const float2*>(&sm.bias[l]);
-          const float2 bu = *reinterpret_cast<const float2*>(&sm.bias[64 + l]);
+        for (int k = 0; k < 8; ++k) {
+          const int l = 16 * qtr + 2 * k;
           const float2 wl = *reinterpret_cast<const float2*>(&sm.wv[l]);
-          pe = ffma2(wl, tanh_times_sigmoid2(fadd2(make_float2(zw[2 * k], zw[2 * k + 1]), bw),
-                                             fadd2(make_float2(zu[2 * k], zu[2 * k + 1]), bu)),
-                     pe);
+          float2 xw = make_float2(zw[2 * k], zw[2 * k + 1]);
+          float2 xu = make_float2(zu[2 * k], zu[2 * k + 1]);
+          if (kBias) {
+            xw = fadd2(xw, *reinterpret_cast<const float2*>(&sm.bias[l]));
+            xu = fadd2(xu, *reinterpret_cast<const float2*>(&sm.bias[64 + l]));
+          }
+          pe = ffma2(wl, tanh_times_sigmoid2(xw, xu), pe);
         }
         e2x += pe.x;
         e2y += pe.y;
@@ -642,12 +654,17 @@ cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_
   if ((e = make_tmap_bf16_2d(&tw, a.W, 64, (uint64_t)a.H * 64, 64, 64, 64)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16_2d(&tu, a.U, 64, (uint64_t)a.H * 64, 64, 64, 64)) != cudaSuccess) return e;
   const int smem = (int)sizeof(PoolTcSmem) + 1024;
-  if ((e = cudaFuncSetAttribute(router_pool_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                smem)) != cudaSuccess)
+  const bool bias = a.bW || a.bU;
+  if ((e = cudaFuncSetAttribute(bias ? router_pool_tc_kernel<true> : router_pool_tc_kernel<false>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
     return e;
   prof_before(VP_KERNEL_ROUTER_POOL, st);
-  router_pool_tc_kernel<<<dim3(pool_split, a.H), kPoolTcThreads, smem, st>>>(tq, tw, tu, a, sc,
-                                                                            pool_split);
+  if (bias)
+    router_pool_tc_kernel<true><<<dim3(pool_split, a.H), kPoolTcThreads, smem, st>>>(tq, tw, tu, a, sc,
+                                                                                    pool_split);
+  else
+    router_pool_tc_kernel<false><<<dim3(pool_split, a.H), kPoolTcThreads, smem, st>>>(tq, tw, tu, a, sc,
+                                                                                     pool_split);
   prof_after(st);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
