@@ -15,10 +15,10 @@
 //                     columns (D1 has been read by then);
 //   y = C + sigma(D2g + b2g) (.) (D2d + b2d), bf16, staged in shared memory (128-byte swizzle)
 //                     and written by a TMA tensor store into Y[:, h, :].
-// A mean tile writes Broadcast(mean of V_h) through the same staging and store.
+// A mean item writes Broadcast(mean of V_h) over 1,024 tokens with coalesced 16-byte stores.
 //
 // Roles (576 threads, one CTA per SM, persistent over items taken kBatch at a time from a
-// device counter: surrogate tiles head-major, then mean tiles):
+// device counter: surrogate tiles of 128 tokens head-major, then mean items of 1,024 tokens):
 //   all        at the start, every surrogate head's per-head vectors into shared memory
 //              (c1 = W1[:, d:] C_h + b1, the second layer's biases, C_h);
 //   warp 0     producer: items, TMA loads of the V tiles (kStages ring) and of each head's
@@ -46,7 +46,8 @@ namespace vp {
 
 namespace {
 
-constexpr int kTcTile = 128;      // tokens per item
+constexpr int kTcTile = 128;      // tokens per surrogate item
+constexpr int kMeanRows = 1024;   // tokens per mean item (a pure write, handed over less often)
 constexpr int kTcStages = 4;      // V tiles in flight
 constexpr int kTcGroups = 2;      // epilogue groups (= TMEM accumulators)
 constexpr int kTcBatch = 4;       // items taken from the counter at a time
@@ -119,7 +120,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
   const int n_surr = __ldg(a.offsets + 2) - s_first, n_mean = s_first - m_first;
   const int T = (a.N + kTcTile - 1) / kTcTile;
   const int surr_items = n_surr * T;
-  const int items = surr_items + n_mean * T;
+  const int Tm = (a.N + kMeanRows - 1) / kMeanRows;  // mean items per head
+  const int items = surr_items + n_mean * Tm;
 
   if (tid == 0) {
     for (int s = 0; s < kTcStages; ++s) {
@@ -231,7 +233,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
         __syncwarp();
         tma_k[st] = k;
       } else {
-        const int slot = (it - surr_items) / T;
+        const int slot = (it - surr_items) / Tm;
         const int h = __ldg(a.head_ids + m_first + slot);
         if (elect_one()) {
           sm.stage_item[st] = it;
@@ -455,7 +457,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
       if (it < 0) break;
       const int h = *reinterpret_cast<volatile int*>(&sm.acc_head[g]);
       const bool surr = it < surr_items;
-      const int tile = (surr ? it : it - surr_items) % T;
+      const int tile = surr ? it % T : (it - surr_items) % Tm;  // a mean item spans kMeanRows rows
       const int slot = surr ? it / T : 0;  // surrogate head slot: its vectors
       const float* c1 = sm.c1[slot];
       const float* b2 = sm.b2[slot];
@@ -492,12 +494,30 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
         ok = mbar_wait_warp(&sm.d2_full[g], sj & 1, err, abort_flag);
         ++sj;
       }
+      if (!surr) {
+        // Broadcast(mean of V_h) straight to Y (no staging: a store pipeline two tiles deep
+        // per SM would hold these pure-write tiles back): eight threads per row, each a 16-byte
+        // chunk, so that a warp writes whole 128-byte rows.
+        ok = group_all(ok, g);
+        if (!ok) break;
+        if (gt == 0) mbar_arrive(&sm.taken[g]);  // every thread has read this tile's item
+        const int jc = gt & 7;
+        const float4 m0 = __ldg(reinterpret_cast<const float4*>(a.mean_v + h * 64) + 2 * jc);
+        const float4 m1 = __ldg(reinterpret_cast<const float4*>(a.mean_v + h * 64) + 2 * jc + 1);
+        const uint4 val = make_uint4(pack_bf16x2(m0.x, m0.y), pack_bf16x2(m0.z, m0.w),
+                                     pack_bf16x2(m1.x, m1.y), pack_bf16x2(m1.z, m1.w));
+        for (int r = gt >> 3; r < kMeanRows; r += kGroupThreads / 8) {
+          const int grow = tile * kMeanRows + r;
+          if (grow < a.N) *(reinterpret_cast<uint4*>(a.y + ((size_t)grow * H + h) * 64) + jc) = val;
+        }
+        continue;
+      }
       // The staging buffer is free once the previous store from it has read it.
       if (gt == 0) tma_store_wait_read<0>();
       ok = group_all(ok, g);
       if (!ok) break;
       if (gt == 0) mbar_arrive(&sm.taken[g]);  // every thread has read this tile's item
-      if (surr) {
+      {
         // y = C + sigma(D2g + b2g) (.) (D2d + b2d) for chunk c of 16 output columns, from
         // D2' = 2 D2: sigma(u) = 1 / (1 + 2^(-log2(e) u)) with the exponent
         // -log2(e) / 2 D2g' + nbg, nbg = -log2(e) b2g held per head.
@@ -535,14 +555,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
           }
         }
         tc_fence_before();
-      } else {  // Broadcast(mean of V_h): this warp's output-column chunks
-        const float4* m = reinterpret_cast<const float4*>(a.mean_v + h * 64);
-        for (int jc = 2 * f0; jc < 2 * f1; ++jc) {
-          const float4 m0 = __ldg(m + 2 * jc), m1 = __ldg(m + 2 * jc + 1);
-          *reinterpret_cast<uint4*>(yrow + ((jc ^ (row & 7)) << 4)) =
-              make_uint4(pack_bf16x2(m0.x, m0.y), pack_bf16x2(m0.z, m0.w), pack_bf16x2(m1.x, m1.y),
-                         pack_bf16x2(m1.z, m1.w));
-        }
       }
       fence_proxy_async_smem();
       group_all(true, g);
