@@ -298,6 +298,23 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
                           void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * vp_global_stack_host -- vp_global_stack for tokens that live in host memory: copies x_in
+ * (HOST pointer, [N][D] bf16) into x_dev (device, [N][D] bf16, caller-owned), runs the
+ * n_layers blocks on x_dev in place, and copies the result to x_out (HOST pointer, [N][D]
+ * bf16; may equal x_in).  Both copies are done by the library's own kernel, which reads and
+ * writes the host memory through its device-visible address, so x_in and x_out must be
+ * page-locked (cudaHostAlloc, cudaHostRegister, or a framework's pinned allocator): other
+ * host memory returns VP_ERR_INVALID_ARG.  Everything is enqueued on `stream` and the call
+ * returns without waiting; x_out is complete once the stream is.  The other arguments are
+ * those of vp_global_stack.  All pointers 16-byte aligned.
+ */
+vp_status vp_global_stack_host(const vp_dims* dims, int32_t n_layers, const vp_bf16* x_in,
+                               vp_bf16* x_out, vp_bf16* x_dev, const vp_layer_weights* layers,
+                               const int32_t* force_modes, int32_t* modes_out, float* s_out,
+                               float* s_attn_out, float ln_eps, void* ws, size_t ws_bytes,
+                               void* stream);
+
+/*
  * vp_router_noalloc -- vp_router without a workspace, for callers that cannot allocate
  * device memory when they call the router (for example a plug-in inside a host framework
  * whose memory pool already reserves the GPU's memory and forbids raw cudaMalloc, or a
@@ -344,7 +361,8 @@ vp_status vp_router_noalloc_error(uint32_t* host_bits, void* stream);
 #define VP_KERNEL_LAYER_NORM 8  /* LayerNorm, and the stack's LN1 statistics pass and QKV
                                    weight fold */
 #define VP_KERNEL_MERGE 9       /* token merging (vp_merge_options) and the unmerge */
-#define VP_KERNEL_CLASSES 10
+#define VP_KERNEL_HOST_COPY 10  /* host <-> device copies of vp_global_stack_host */
+#define VP_KERNEL_CLASSES 11
 
 /*
  * Launch profiler (for benchmarks; not part of the method).  Between vp_profile_begin and

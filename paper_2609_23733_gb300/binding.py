@@ -22,7 +22,7 @@ VP_ACT_NONE, VP_ACT_GELU = 0, 1
 VP_DEVERR_WAIT_TIMEOUT, VP_DEVERR_NAN_SALIENCY = 1, 2
 VP_VARIANT_MEAN_QPOOL, VP_VARIANT_MEAN_CONTEXT, VP_VARIANT_NO_RESIDUAL, VP_VARIANT_LINEAR_ATTENTION = 1, 2, 4, 8
 KERNEL_CLASSES = ["gemm", "router_pool", "router_keys", "router_r", "bin_heads", "attn_full",
-                  "surrogate", "mean", "layer_norm", "merge"]
+                  "surrogate", "mean", "layer_norm", "merge", "host_copy"]
 
 STATUS = {0: "VP_OK", 1: "VP_ERR_INVALID_ARG", 2: "VP_ERR_UNSUPPORTED_SHAPE", 3: "VP_ERR_ALIGNMENT",
           4: "VP_ERR_CUDA", 5: "VP_ERR_DEVICE_TIMEOUT", 6: "VP_ERR_WORKSPACE",
@@ -96,6 +96,9 @@ _SIGS = [
                                           c_void_p, c_void_p,
                                           c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
                                           c_void_p]),
+    ("vp_global_stack_host", c_int32, [POINTER(VpDims), c_int32, c_void_p, c_void_p, c_void_p,
+                                       POINTER(VpLayerWeights), c_void_p, c_void_p, c_void_p, c_void_p,
+                                       c_float, c_void_p, c_size_t, c_void_p]),
     ("vp_profile_begin", c_int32, [c_int32]),
     ("vp_profile_end", c_int32, [POINTER(c_int32), POINTER(c_int32), POINTER(c_float)]),
     ("vp_global_stack", c_int32, [POINTER(VpDims), c_int32, c_void_p, POINTER(VpLayerWeights),
@@ -135,6 +138,15 @@ def _p(t):
             raise ValueError("tensors must be contiguous")
         return t.data_ptr()
     return int(t)
+
+
+def _host_p(t):
+    """Address of a page-locked, contiguous CPU tensor (a host buffer the GPU can reach)."""
+    if not isinstance(t, torch.Tensor) or t.device.type != "cpu":
+        raise ValueError("a CPU tensor is required")
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    return t.data_ptr()
 
 
 def _stream(stream=None):
@@ -325,6 +337,16 @@ def vp_global_stack(dm, x_inout, layers, force_modes, modes_out, s_out, ln_eps, 
     _check(lib().vp_global_stack(ctypes.byref(dm), len(layers), _p(x_inout), arr, _p(force_modes),
                                  _p(modes_out), _p(s_out), _p(s_attn_out), float(ln_eps), _p(ws), ws.numel(),
                                  _stream(stream)), "vp_global_stack")
+
+
+def vp_global_stack_host(dm, x_in, x_out, x_dev, layers, force_modes, modes_out, s_out, ln_eps, ws,
+                         stream=None, s_attn_out=None):
+    """vp_global_stack on tokens in page-locked host memory (x_in, x_out: pinned CPU tensors);
+    x_dev is the device buffer the blocks run on."""
+    arr = (VpLayerWeights * len(layers))(*layers)
+    _check(lib().vp_global_stack_host(ctypes.byref(dm), len(layers), _host_p(x_in), _host_p(x_out), _p(x_dev), arr,
+                                      _p(force_modes), _p(modes_out), _p(s_out), _p(s_attn_out), float(ln_eps),
+                                      _p(ws), ws.numel(), _stream(stream)), "vp_global_stack_host")
 
 
 def vp_profile_begin(max_launches: int):

@@ -615,10 +615,11 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
                    qkv, y, s_out, s_attn_out, modes_out, sc, st, nullptr, &qa);
 }
 
-vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
-                          const vp_layer_weights* layers, const int32_t* force_modes,
-                          int32_t* modes_out, float* s_out, float* s_attn_out, float ln_eps,
-                          void* ws, size_t ws_bytes, void* stream) {
+// The host-side checks of vp_global_stack (also run by vp_global_stack_host before it
+// enqueues anything); *any_merge: some block merges tokens.
+static vp_status check_stack(const vp_dims* dims, int32_t n_layers, const vp_bf16* x_inout,
+                             const vp_layer_weights* layers, size_t ws_bytes, const void* ws,
+                             bool* any_merge_out) {
   VP_TRY(check_dims(dims));
   if (n_layers < 1 || !x_inout || !layers) return VP_ERR_INVALID_ARG;
   if (!aligned16(x_inout)) return VP_ERR_ALIGNMENT;
@@ -645,7 +646,17 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
   }
   if (!ws || ws_bytes < (any_merge ? stack_merge_ws_bytes(dims) : stack_ws_bytes(dims)))
     return VP_ERR_WORKSPACE;
-  VP_TRY(check_device());
+  *any_merge_out = any_merge;
+  return check_device();
+}
+
+vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inout,
+                          const vp_layer_weights* layers, const int32_t* force_modes,
+                          int32_t* modes_out, float* s_out, float* s_attn_out, float ln_eps,
+                          void* ws, size_t ws_bytes, void* stream) {
+  bool any_merge = false;
+  VP_TRY(check_stack(dims, n_layers, x_inout, layers, ws_bytes, ws, &any_merge));
+  const int D = dims->H * kHeadDim;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t N = dims->N;
   RouterScratch sc = carve_router_scratch(ws, dims->H);
@@ -776,6 +787,40 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     VP_TRY(from_cuda(launch_linear(f2, sms, st)));
   }
   return VP_OK;
+}
+
+// A host pointer the GPU can read and write (page-locked), as a device-visible address.
+static vp_status device_view_of_host(const void* p, void** dev) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();  // clear the error of an unknown pointer
+    return VP_ERR_INVALID_ARG;
+  }
+  if (at.type != cudaMemoryTypeHost || !at.devicePointer) return VP_ERR_INVALID_ARG;
+  *dev = at.devicePointer;
+  return VP_OK;
+}
+
+vp_status vp_global_stack_host(const vp_dims* dims, int32_t n_layers, const vp_bf16* x_in,
+                               vp_bf16* x_out, vp_bf16* x_dev, const vp_layer_weights* layers,
+                               const int32_t* force_modes, int32_t* modes_out, float* s_out,
+                               float* s_attn_out, float ln_eps, void* ws, size_t ws_bytes,
+                               void* stream) {
+  if (!x_in || !x_out || !x_dev) return VP_ERR_INVALID_ARG;
+  if (!aligned16(x_in) || !aligned16(x_out)) return VP_ERR_ALIGNMENT;
+  bool any_merge = false;
+  VP_TRY(check_stack(dims, n_layers, x_dev, layers, ws_bytes, ws, &any_merge));
+  void* in_dev = nullptr;
+  void* out_dev = nullptr;
+  VP_TRY(device_view_of_host(x_in, &in_dev));
+  VP_TRY(device_view_of_host(x_out, &out_dev));
+  const size_t bytes = (size_t)dims->N * dims->H * kHeadDim * sizeof(vp_bf16);  // a multiple of 16
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int sms = device_sm_count();
+  VP_TRY(from_cuda(launch_host_copy(in_dev, x_dev, bytes, sms, st)));
+  VP_TRY(vp_global_stack(dims, n_layers, x_dev, layers, force_modes, modes_out, s_out, s_attn_out,
+                         ln_eps, ws, ws_bytes, stream));
+  return from_cuda(launch_host_copy(x_dev, out_dev, bytes, sms, st));
 }
 
 }  // extern "C"

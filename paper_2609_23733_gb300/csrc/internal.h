@@ -232,6 +232,11 @@ cudaError_t launch_unmerge_ln(int N, int D, const int* assign, const __nv_bfloat
                               const float* ls, const float* g, const float* b, float eps,
                               __nv_bfloat16* x, __nv_bfloat16* z, cudaStream_t st);
 
+// Copy of `bytes` (a multiple of 16; both addresses 16-byte aligned and device-visible, e.g.
+// pinned host memory) by the SMs (host_copy.cu).
+cudaError_t launch_host_copy(const void* src, void* dst, size_t bytes, int num_sms,
+                             cudaStream_t st);
+
 // One warp waiting on an mbarrier that never completes, bounded by limit_ns (self-test of the
 // wait limit; sets VP_DEVERR_WAIT_TIMEOUT in *err).
 cudaError_t launch_wait_selftest(unsigned int* err, unsigned long long limit_ns, cudaStream_t st);

@@ -95,6 +95,11 @@ def test_host_side_validation(vp):
     assert na(dm, q=A + 8) == 3
     # its error reader needs somewhere to write the bits
     assert lib.vp_router_noalloc_error(None, None) == 1
+    # vp_global_stack_host: missing buffers, misaligned host buffers (before any device query)
+    hs = lambda a, b, c: lib.vp_global_stack_host(ctypes.byref(dm), 1, a, b, c, None, None, None, None, None,
+                                                  ctypes.c_float(1e-6), A, 1 << 30, None)
+    assert hs(None, A, A) == 1 and hs(A, None, A) == 1 and hs(A, A, None) == 1
+    assert hs(A + 8, A, A) == 3 and hs(A, A + 4, A) == 3
     # vp_linear: shapes and alignment
     assert lib.vp_linear(100, 12, 64, A, A, None, 0, None, None, A, None) == 2
     assert lib.vp_linear(100, 256, 60, A, A, None, 0, None, None, A, None) == 2

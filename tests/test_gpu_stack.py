@@ -47,6 +47,40 @@ def _run_stack(x_bits, ws_host, N, force=None, H=16):
     return _f64(x), modes.cpu().numpy(), s.cpu().numpy()
 
 
+def test_stack_host_buffers_equal_the_device_path():
+    """vp_global_stack_host (tokens in page-locked host memory, copied by the library's own
+    kernel both ways) gives the bits of vp_global_stack on a device copy of the tokens, in
+    place (x_out = x_in) and into a second buffer; unpinned host memory is refused."""
+    N, L, H = 1000, 2, 16
+    g = synth.rng(41)
+    wts = [synth.make_layer_weights(g, block=True, bias_std=0.05) for _ in range(L)]
+    x_bits = synth.make_tokens(41, N)
+    force = np.array([synth.forced_mix(H, f) for f in (0.25, 0.0)])
+    dm = vpb.dims(N, H)
+    dws = [vpb.to_device(w) for w in wts]
+    layers = [vpb.layer_weights(w) for w in dws]
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK)
+    fm = torch.tensor(force, device="cuda")
+    modes = torch.zeros(L, H, dtype=torch.int32, device="cuda")
+    s = torch.zeros(L, H, device="cuda")
+    x = vpb.bf16_from_bits(x_bits)
+    vpb.vp_global_stack(dm, x, layers, fm, modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    want = x.cpu()
+    host_in = vpb.bf16_from_bits(x_bits).cpu().pin_memory()
+    host_out = torch.zeros_like(host_in).pin_memory()
+    x_dev = torch.empty(N, H * 64, dtype=torch.bfloat16, device="cuda")
+    for out in (host_out, host_in):  # into a second buffer, then in place
+        vpb.vp_global_stack_host(dm, host_in, out, x_dev, layers, fm, modes, s, 1e-6, ws)
+        torch.cuda.synchronize()
+        assert vpb.vp_read_device_error(ws) == 0
+        assert torch.equal(out, want)
+    pageable = vpb.bf16_from_bits(x_bits).cpu()
+    with pytest.raises(vpb.VPError) as e:
+        vpb.vp_global_stack_host(dm, pageable, host_out, x_dev, layers, fm, modes, s, 1e-6, ws)
+    assert e.value.status == 1  # VP_ERR_INVALID_ARG: not page-locked
+
+
 def test_stack_three_blocks_all_modes():
     N, L = 600, 3
     g = synth.rng(5)
