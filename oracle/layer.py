@@ -153,7 +153,7 @@ def global_block(X, lw, force_modes=None, materialize=round_bf16, eps=LN_EPS,
     if merge is not None:
         row_of, dst_tok = destinations(X.shape[0], merge["tokens_per_view"], merge["patch_start"],
                                        merge["stride"])
-        own, scores = match(key_metric(Xt, lw, mat), row_of, dst_tok)
+        own, scores = match(key_metric(Xt, lw), row_of, dst_tok)
         asg = own if assign is None else np.asarray(assign)
         Xm = mat(merge_tokens(Xt, asg, len(dst_tok)))
         att = moh_attention(Xm, lw, force_modes=force_modes, materialize=materialize, tau_low=tau_low,

@@ -26,16 +26,17 @@ def destinations(N: int, tokens_per_view: int, patch_start: int, stride: int):
     return row_of, dst_tok
 
 
-def key_metric(Xt, lw, materialize):
-    """Unit head-mean keys.  Storage points of the library: the head-mean key weights, the
-    metric rows and the unit rows are bf16 (materialize)."""
+def key_metric(Xt, lw):
+    """Unit head-mean keys of the LN1 output, in exact arithmetic: k_i = mean_h (Xt_i W_K,h^T
+    + b_K,h), m_i = k_i / |k_i| (0 for a zero key).  The metric is no storage point of the
+    block (the paper fixes no precision for it), so nothing here is rounded to bf16."""
     H = lw["r_W"].shape[0]
     D = Xt.shape[1]
     wk = lw["w_qkv"][D:2 * D].reshape(H, 64, D)
     bk = lw["b_qkv"][D:2 * D].reshape(H, 64)
-    k = materialize(np.asarray(Xt, np.float64) @ materialize(wk.mean(axis=0)).T + bk.mean(axis=0))
+    k = np.asarray(Xt, np.float64) @ wk.mean(axis=0).T + bk.mean(axis=0)
     norm = np.sqrt(np.sum(k * k, axis=1, keepdims=True))
-    return materialize(np.where(norm > 0, k / np.where(norm > 0, norm, 1.0), 0.0))
+    return np.where(norm > 0, k / np.where(norm > 0, norm, 1.0), 0.0)
 
 
 def match(m, row_of, dst_tok):

@@ -46,7 +46,7 @@ def test_key_metric_is_the_unit_head_mean_of_the_keys():
     g = synth.rng(4)
     w = oracle.load_layer(synth.make_layer_weights(g, bias_std=0.05))
     x = np.random.default_rng(4).standard_normal((30, 1024))
-    m = oracle.key_metric(x, w, lambda a: np.asarray(a, np.float64))
+    m = oracle.key_metric(x, w)
     k = oracle.qkv_projection(x, w, materialize=None)[:, 1].mean(axis=1)  # [N, d]
     np.testing.assert_allclose(m, k / np.linalg.norm(k, axis=1, keepdims=True), rtol=1e-10, atol=1e-12)
 
