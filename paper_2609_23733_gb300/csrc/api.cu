@@ -201,11 +201,12 @@ size_t stack_ws_bytes(const vp_dims* dm) {
 }
 
 // Token-merging scratch (vp_merge_options): metric weights and rows, the destination and
-// membership tables, the merged tokens and their attention output.
+// membership tables, the merged tokens and their attention output (whose region holds the
+// partial sums of the merged tokens before the attention writes it).
 size_t merge_scratch_bytes(size_t N, size_t D) {
   return align_up(64 * D * 2) + align_up(64 * sizeof(float)) + 3 * align_up(N * 64 * 2) +
          7 * align_up((N + 1) * sizeof(int)) + align_up(N * sizeof(unsigned long long)) +
-         2 * align_up(N * D * 2);
+         align_up(N * D * 2) + align_up(std::max(N * D * 2, merge_slot_bytes(N, D)));
 }
 
 size_t stack_merge_ws_bytes(const vp_dims* dm) {
@@ -706,6 +707,7 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
     ms.err = sc.err;
   }
   __nv_bfloat16* merged_out = any_merge ? reinterpret_cast<__nv_bfloat16*>(p) : nullptr;  // [Np][D]
+  ms.slots = reinterpret_cast<float*>(merged_out);  // free until the block's attention writes it
   __nv_bfloat16* x = reinterpret_cast<__nv_bfloat16*>(x_inout);
   const int sms = device_sm_count();
   VP_TRY(from_cuda(launch_ln_partials(dims->N, D, x, part, st)));

@@ -208,8 +208,11 @@ struct MergeScratch {
   int* members;          // [N]
   unsigned long long* best;  // [Ns] matching: (score, destination) keys, 0 before the matching
   __nv_bfloat16* xm;     // [Np][D] merged tokens
+  float* slots;          // [ceil(N / 32)][2][D] partial sums of the merged tokens (merge means)
   unsigned int* err;
 };
+// Bytes of MergeScratch::slots for N tokens of D channels.
+inline size_t merge_slot_bytes(size_t N, size_t D) { return (N + 31) / 32 * 2 * D * sizeof(float); }
 // LN1 of the merging, folded (its output is never stored): the row statistics of x and the
 // scratch of the folded metric weights.
 struct MergeLn {

@@ -103,9 +103,9 @@ __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_b
 //               of two 256-column fp32 accumulators (the epilogue of one chunk overlaps the
 //               MMAs of the next);
 //   warps 4-19  argmax: a source row (TMEM lane) and a quarter of each chunk's columns per
-//               thread, loaded into registers (two tcgen05.ld of 32 columns) before the
-//               accumulator is released, so that the max trees overlap the next MMAs.  A tree gives
-//               the piece's max; a piece whose max beats the row's best is copied to the
+//               thread, loaded into registers (two tcgen05.ld.red of 32 columns, which also
+//               return each 32-column piece's maximum) before the accumulator is released; a
+//               piece whose max beats the row's best is copied to the
 //               thread's slot in shared memory, and the column is looked up there once, at the
 //               end of the segment.  Chunks ascend within a segment, so the first piece that
 //               reaches a score holds its lowest column.
@@ -295,28 +295,30 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
         const int valid = g.Np - c0;                 // columns past it hold no destination
         // Both pieces into registers, then the accumulator goes back to the MMA warp at once:
         // the max trees below overlap the next chunks' MMAs.
-        float v[kCols / 32][32];
+        // Each piece's maximum comes with its load (tcgen05.ld.red).
+        float v[kCols / 32][32], pm[kCols / 32];
 #pragma unroll
-        for (int p = 0; p < kCols / 32; ++p) tmem_ld32(t_lane + ab * kMatchN + 32 * p, v[p]);
+        for (int p = 0; p < kCols / 32; ++p) tmem_ld32_max(t_lane + ab * kMatchN + 32 * p, v[p], pm[p]);
         tmem_wait_ld();
         tc_fence_before();
         mbar_arrive(&sm.acc_empty[ab]);
 #pragma unroll
         for (int p = 0; p < kCols / 32; ++p) {
           float* x = v[p];
-          if (32 * p + 32 > valid) {
+          float mx = pm[p];
+          if (32 * p + 32 > valid) {  // columns past the last destination: masked, then a tree
 #pragma unroll
             for (int k = 0; k < 32; ++k)
               if (32 * p + k >= valid) x[k] = -INFINITY;
+            float q[4];  // four independent 3-input max chains, then a short tree
+#pragma unroll
+            for (int k = 0; k < 4; ++k) q[k] = fmaxf(x[k], x[k + 4]);
+#pragma unroll
+            for (int k = 8; k < 32; k += 8)
+#pragma unroll
+              for (int e = 0; e < 4; ++e) q[e] = fmax3(q[e], x[k + e], x[k + 4 + e]);
+            mx = fmax3(q[0], q[1], fmaxf(q[2], q[3]));
           }
-          float q[4];  // four independent 3-input max chains, then a short tree
-#pragma unroll
-          for (int k = 0; k < 4; ++k) q[k] = fmaxf(x[k], x[k + 4]);
-#pragma unroll
-          for (int k = 8; k < 32; k += 8)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) q[e] = fmax3(q[e], x[k + e], x[k + 4 + e]);
-          const float mx = fmax3(q[0], q[1], fmaxf(q[2], q[3]));
           if (mx > bv) {  // a strictly better piece: keep its scores
             bv = mx;
             bcol = c0 + 32 * p;
@@ -436,67 +438,24 @@ __global__ void merge_fill_kernel(int N, const int* assign, const int* offs, int
   members[offs[r] + atomicAdd(fill + r, 1)] = i;
 }
 
-// One warp per merged token: the mean of its members' rows of LN1(x), normalised on the fly
-// (the LN1 output is not stored): for each member, its mean and 1 / sqrt(var + eps) from the
+// The merged tokens: the mean of each merged row's members' rows of LN1(x), normalised on the
+// fly (the LN1 output is not stored): per member, its mean and 1 / sqrt(var + eps) from the
 // (mean, M2) of its 128-column blocks, then (x - mu) rstd summed in fp32; at the end
-// gamma (.) sum / count + beta (D = 256 C; lane l holds 16-byte chunks c 32 + l).
+// gamma (.) sum / count + beta.  The member list (grouped by merged row) is cut into chunks of
+// kMeanChunk consecutive entries, one warp each, so that every warp reads the same number of
+// rows however unevenly the sources chose their destinations (later blocks put hundreds of
+// sources on a few destinations).  A merged row whose members all lie in the chunk is written
+// there.  A row that crosses a chunk boundary leaves its chunk's part of the sum in a slot
+// (slot 1 of its first chunk, slot 0 of every later one) and counts its members off fill[r],
+// which holds the row's member count; the chunk that brings it to 0 adds the row's slots in
+// chunk order and writes the mean.  D = 256 C; lane l holds 16-byte chunks c 32 + l.
+constexpr int kMeanChunk = 32;
+static_assert(kMeanChunk == 32, "merge_slot_bytes counts chunks of 32 entries");
+
 template <int C>
-__global__ void __launch_bounds__(256, C <= 4 ? 3 : 1)
-    merge_mean_kernel(int Np, const __nv_bfloat16* x, const float2* part, const float* gamma,
-                      const float* beta, float eps, const int* offs, const int* members,
-                      __nv_bfloat16* xm) {
-  constexpr int D = 256 * C, NB = D / 128;  // 128-column blocks of a row (NB <= 32)
-  const int lane = threadIdx.x & 31;
-  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (r >= Np) return;
-  const int b = offs[r], e = offs[r + 1];
-  float acc[C][8];
-#pragma unroll
-  for (int c = 0; c < C; ++c)
-#pragma unroll
-    for (int k = 0; k < 8; ++k) acc[c][k] = 0.f;
-  // Member indices 32 at a time (one coalesced load), then their rows and statistics, two
-  // members in flight.
-  for (int q0 = b; q0 < e; q0 += 32) {
-    const int mine = q0 + lane < e ? members[q0 + lane] : 0;
-    const int nm = min(32, e - q0);
-    for (int k = 0; k < nm; k += 2) {  // two rows' loads issued before any arithmetic
-      uint4 u[2][C];
-      float2 ps[2];
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int i = __shfl_sync(0xffffffffu, mine, min(k + j, nm - 1));
-#pragma unroll
-        for (int c = 0; c < C; ++c)
-          u[j][c] = __ldg(reinterpret_cast<const uint4*>(x + (size_t)i * D + (c * 32 + lane) * 8));
-        ps[j] = lane < NB ? __ldg(part + (size_t)i * NB + lane) : make_float2(0.f, 0.f);
-      }
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        if (k + j >= nm) break;  // uniform across the warp
-        float sm = ps[j].x;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
-        const float mu = sm / (float)NB;
-        const float d = ps[j].x - mu;
-        float m2 = lane < NB ? ps[j].y + 128.f * d * d : 0.f;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) m2 += __shfl_xor_sync(0xffffffffu, m2, o);
-        const float rstd = rsqrtf(m2 / (float)D + eps);
-        const float nmr = -mu * rstd;
-#pragma unroll
-        for (int c = 0; c < C; ++c) {
-          const uint32_t w[4] = {u[j][c].x, u[j][c].y, u[j][c].z, u[j][c].w};
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {
-            acc[c][2 * kk] += fmaf(bf16_lo(w[kk]), rstd, nmr);
-            acc[c][2 * kk + 1] += fmaf(bf16_hi(w[kk]), rstd, nmr);
-          }
-        }
-      }
-    }
-  }
-  const float inv = 1.f / (float)(e - b);
+__device__ __forceinline__ void store_mean(const float (&acc)[C][8], float inv, int lane,
+                                           const float* gamma, const float* beta,
+                                           __nv_bfloat16* dst) {
 #pragma unroll
   for (int c = 0; c < C; ++c) {
     const int col = (c * 32 + lane) * 8;
@@ -511,7 +470,129 @@ __global__ void __launch_bounds__(256, C <= 4 ? 3 : 1)
     o.y = pack_bf16x2(fmaf(gg[2], acc[c][2] * inv, bb[2]), fmaf(gg[3], acc[c][3] * inv, bb[3]));
     o.z = pack_bf16x2(fmaf(gg[4], acc[c][4] * inv, bb[4]), fmaf(gg[5], acc[c][5] * inv, bb[5]));
     o.w = pack_bf16x2(fmaf(gg[6], acc[c][6] * inv, bb[6]), fmaf(gg[7], acc[c][7] * inv, bb[7]));
-    *reinterpret_cast<uint4*>(xm + (size_t)r * D + col) = o;
+    *reinterpret_cast<uint4*>(dst + col) = o;
+  }
+}
+
+// The members [a, b) of the chunk (entries q0 + a .. q0 + b - 1 of the list) that belong to
+// merged row r, summed in acc: the row's mean if the chunk holds all of its members, else the
+// chunk's slot and the count-off described above.
+template <int C>
+__device__ __forceinline__ void flush_row(float (&acc)[C][8], int r, int a, int b, int ch, int q0,
+                                          int nm, int lane, const int* offs, int* fill,
+                                          float* slots, const float* gamma, const float* beta,
+                                          __nv_bfloat16* xm) {
+  constexpr int D = 256 * C;
+  const int first = __ldg(offs + r), last = __ldg(offs + r + 1);
+  if (first < q0 || last > q0 + nm) {  // the row crosses a chunk boundary
+    float* slot = slots + ((size_t)ch * 2 + (first < q0 ? 0 : 1)) * D;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      float4* d = reinterpret_cast<float4*>(slot + (c * 32 + lane) * 8);
+      d[0] = make_float4(acc[c][0], acc[c][1], acc[c][2], acc[c][3]);
+      d[1] = make_float4(acc[c][4], acc[c][5], acc[c][6], acc[c][7]);
+    }
+    __threadfence();
+    __syncwarp();
+    int done = 0;
+    if (lane == 0) done = atomicSub(fill + r, b - a) == b - a;
+    if (!__shfl_sync(0xffffffffu, done, 0)) return;  // another chunk of the row finishes it
+    __threadfence();
+    const int c0 = first / kMeanChunk, c1 = (last - 1) / kMeanChunk;
+#pragma unroll
+    for (int c = 0; c < C; ++c)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[c][k] = 0.f;
+#pragma unroll 1
+    for (int cc = c0; cc <= c1; ++cc) {
+      const float* sl = slots + ((size_t)cc * 2 + (cc == c0 ? 1 : 0)) * D;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const float4* q = reinterpret_cast<const float4*>(sl + (c * 32 + lane) * 8);
+        const float4 u0 = __ldcg(q), u1 = __ldcg(q + 1);
+        acc[c][0] += u0.x;
+        acc[c][1] += u0.y;
+        acc[c][2] += u0.z;
+        acc[c][3] += u0.w;
+        acc[c][4] += u1.x;
+        acc[c][5] += u1.y;
+        acc[c][6] += u1.z;
+        acc[c][7] += u1.w;
+      }
+    }
+  }
+  store_mean<C>(acc, 1.f / (float)(last - first), lane, gamma, beta, xm + (size_t)r * D);
+}
+
+// Two CTAs per SM at D = 1,024: the accumulator, two rows in flight and the slot path fit in
+// 128 registers without spills (three CTAs spill and measured 1 ms slower per S = 100 forward).
+template <int C>
+__global__ void __launch_bounds__(256, C <= 2 ? 3 : (C <= 4 ? 2 : 1))
+    merge_mean_kernel(int N, const __nv_bfloat16* x, const float2* part, const float* gamma,
+                      const float* beta, float eps, const int* offs, const int* members,
+                      const int* assign, int* fill, float* slots, __nv_bfloat16* xm) {
+  constexpr int D = 256 * C, NB = D / 128;  // 128-column blocks of a row (NB <= 32)
+  const int lane = threadIdx.x & 31;
+  const int ch = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int q0 = ch * kMeanChunk;
+  if (q0 >= N) return;
+  const int nm = min(kMeanChunk, N - q0);
+  const int mine = lane < nm ? __ldg(members + q0 + lane) : 0;  // one coalesced load
+  const int my_row = lane < nm ? __ldg(assign + mine) : -1;
+  float acc[C][8];
+#pragma unroll
+  for (int c = 0; c < C; ++c)
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[c][k] = 0.f;
+  int cur = __shfl_sync(0xffffffffu, my_row, 0), run0 = 0;  // the current row and its first entry
+  // Entries 0 .. nm - 1, then a sentinel entry nm that ends the last row (one flush site).
+  for (int k = 0; k <= nm; k += 2) {  // two rows' loads issued before any arithmetic
+    uint4 u[2][C];
+    float2 ps[2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int i = __shfl_sync(0xffffffffu, mine, min(k + j, nm - 1));
+#pragma unroll
+      for (int c = 0; c < C; ++c)
+        u[j][c] = __ldg(reinterpret_cast<const uint4*>(x + (size_t)i * D + (c * 32 + lane) * 8));
+      ps[j] = lane < NB ? __ldg(part + (size_t)i * NB + lane) : make_float2(0.f, 0.f);
+    }
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int e = k + j;
+      if (e > nm) break;  // uniform across the warp
+      const int re = __shfl_sync(0xffffffffu, my_row, min(e, nm - 1));
+      const int r = e < nm ? re : -1;
+      if (r != cur) {  // the entries of row cur end here
+        flush_row<C>(acc, cur, run0, e, ch, q0, nm, lane, offs, fill, slots, gamma, beta, xm);
+#pragma unroll
+        for (int c = 0; c < C; ++c)
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) acc[c][kk] = 0.f;
+        cur = r;
+        run0 = e;
+      }
+      if (e == nm) break;
+      float sm = ps[j].x;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+      const float mu = sm / (float)NB;
+      const float d = ps[j].x - mu;
+      float m2 = lane < NB ? ps[j].y + 128.f * d * d : 0.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) m2 += __shfl_xor_sync(0xffffffffu, m2, o);
+      const float rstd = rsqrtf(m2 / (float)D + eps);
+      const float nmr = -mu * rstd;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t w[4] = {u[j][c].x, u[j][c].y, u[j][c].z, u[j][c].w};
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          acc[c][2 * kk] += fmaf(bf16_lo(w[kk]), rstd, nmr);
+          acc[c][2 * kk + 1] += fmaf(bf16_hi(w[kk]), rstd, nmr);
+        }
+      }
+    }
   }
 }
 
@@ -674,13 +755,17 @@ cudaError_t launch_merge_prepare(const MergeGeo& g, int H, const __nv_bfloat16* 
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   prof_before(VP_KERNEL_MERGE, st);
-  const int grid = (g.Np + 7) / 8;
+  const int grid = ((g.N + kMeanChunk - 1) / kMeanChunk + 7) / 8;  // a warp per chunk
+#define VP_MEAN(C_)                                                                              \
+  merge_mean_kernel<C_><<<grid, 256, 0, st>>>(g.N, x, ln.part, ln.g, ln.b, ln.eps, s.offs,       \
+                                              s.members, s.assign, s.fill, s.slots, s.xm)
   switch (D / 256) {
-    case 1: merge_mean_kernel<1><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
-    case 2: merge_mean_kernel<2><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
-    case 3: merge_mean_kernel<3><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
-    case 4: merge_mean_kernel<4><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
-    case 8: merge_mean_kernel<8><<<grid, 256, 0, st>>>(g.Np, x, ln.part, ln.g, ln.b, ln.eps, s.offs, s.members, s.xm); break;
+    case 1: VP_MEAN(1); break;
+    case 2: VP_MEAN(2); break;
+    case 3: VP_MEAN(3); break;
+    case 4: VP_MEAN(4); break;
+    case 8: VP_MEAN(8); break;
+#undef VP_MEAN
     default: prof_after(st); return cudaErrorInvalidValue;
   }
   prof_after(st);

@@ -188,3 +188,40 @@ def test_matching_ties_go_to_the_lowest_destination():
         assert got[i] == want, (int(i), int(got[i]), want)
         n_ties += int(cls.sum() > 1)
     assert n_ties >= 20, n_ties
+
+
+@pytest.mark.parametrize("stride", [4, 10])
+def test_one_destination_takes_most_sources(stride):
+    """Every source of views 1-3 is view 0's token 100 plus its own noise, so all of them join
+    merged row 100 (a clear winner): one merged token of 577 (stride 4) or 691 (stride 10)
+    distinct members, whose entries of the member list span many of the merge-means kernel's
+    32-entry chunks (partial sums in slots, finished by the last chunk), beside rows of a single
+    member; the block output is checked against the oracle with the library's matching."""
+    N = 4 * P224
+    g = synth.rng(25)
+    w = synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1)
+    x_bits = synth.make_tokens(25, N)
+    row_of, _ = oracle.destinations(N, P224, 5, stride)
+    src = np.nonzero(row_of < 0)[0]
+    base = synth.bf16_bits_to_f32(x_bits[100])
+    noise = np.random.default_rng(25).standard_normal((len(src), x_bits.shape[1])).astype(np.float32)
+    x_bits[src] = synth.f32_to_bf16_bits(base[None, :] + 0.1 * noise)
+    force = np.array([[2, 1, 0, 1] * 4])
+    dm = vpb.dims(N, 16)
+    assign = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    dw = vpb.to_device(w)
+    layers = [vpb.layer_weights(dw, None, vpb.merge_options(stride, P224, 5, assign))]
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
+    x = vpb.bf16_from_bits(x_bits)
+    modes = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
+    s = torch.zeros(1, 16, device="cuda")
+    vpb.vp_global_stack(dm, x, layers, torch.tensor(force, dtype=torch.int32, device="cuda"), modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    got = assign.cpu().numpy().astype(np.int64)
+    assert np.all(got[src] == 100)
+    merge = [{"stride": stride, "tokens_per_view": P224, "patch_start": 5}]
+    want, infos = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w)], force_modes=force,
+                                      merge=merge, assign=[got])
+    _check_matching(got, infos[0], "one heavy destination")
+    compare(_f64(x), want, rel=BF16_STEP, what=f"block with a merged token of {len(src) + 1} members")
