@@ -451,6 +451,7 @@ __global__ void merge_fill_kernel(int N, const int* assign, const int* offs, int
 // chunk order and writes the mean.  D = 256 C; lane l holds 16-byte chunks c 32 + l.
 constexpr int kMeanChunk = 32;
 static_assert(kMeanChunk == 32, "merge_slot_bytes counts chunks of 32 entries");
+constexpr int kMeanInFlight = 2;  // member rows whose loads are in flight together
 
 template <int C>
 __device__ __forceinline__ void store_mean(const float (&acc)[C][8], float inv, int lane,
@@ -546,11 +547,11 @@ __global__ void __launch_bounds__(256, C <= 2 ? 3 : (C <= 4 ? 2 : 1))
     for (int k = 0; k < 8; ++k) acc[c][k] = 0.f;
   int cur = __shfl_sync(0xffffffffu, my_row, 0), run0 = 0;  // the current row and its first entry
   // Entries 0 .. nm - 1, then a sentinel entry nm that ends the last row (one flush site).
-  for (int k = 0; k <= nm; k += 2) {  // two rows' loads issued before any arithmetic
-    uint4 u[2][C];
-    float2 ps[2];
+  for (int k = 0; k <= nm; k += kMeanInFlight) {  // the rows' loads issued before any arithmetic
+    uint4 u[kMeanInFlight][C];
+    float2 ps[kMeanInFlight];
 #pragma unroll
-    for (int j = 0; j < 2; ++j) {
+    for (int j = 0; j < kMeanInFlight; ++j) {
       const int i = __shfl_sync(0xffffffffu, mine, min(k + j, nm - 1));
 #pragma unroll
       for (int c = 0; c < C; ++c)
@@ -558,7 +559,7 @@ __global__ void __launch_bounds__(256, C <= 2 ? 3 : (C <= 4 ? 2 : 1))
       ps[j] = lane < NB ? __ldg(part + (size_t)i * NB + lane) : make_float2(0.f, 0.f);
     }
 #pragma unroll
-    for (int j = 0; j < 2; ++j) {
+    for (int j = 0; j < kMeanInFlight; ++j) {
       const int e = k + j;
       if (e > nm) break;  // uniform across the warp
       const int re = __shfl_sync(0xffffffffu, my_row, min(e, nm - 1));

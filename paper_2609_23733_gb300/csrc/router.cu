@@ -103,7 +103,10 @@ __device__ __forceinline__ void pool_finish(const RouterArgs& a, const RouterScr
 //            sum p q), which pool_finish combines over the CTAs of the head.
 constexpr int kPoolTcStages = 4;
 constexpr int kPoolTcThreads = 192;
-constexpr uint32_t kPoolTcTmemCols = 256;
+constexpr int kPoolAccBufs = 2;    // 128-column fp32 accumulators per CTA
+constexpr int kPoolCtasPerSm = 2;  // TMEM: kPoolCtasPerSm x kPoolAccBufs x 128 <= 512 columns
+constexpr uint32_t kPoolTcTmemCols = 128 * kPoolAccBufs;
+static_assert(kPoolCtasPerSm * kPoolTcTmemCols <= 512, "TMEM columns");
 
 struct PoolTcSmem {
   __nv_bfloat16 q[kPoolTcStages][128 * 64];
@@ -113,7 +116,7 @@ struct PoolTcSmem {
   float red_m[4], red_l[4];
   float red_acc[4][64];
   uint64_t q_full[kPoolTcStages], q_empty[kPoolTcStages];
-  uint64_t wu_full, acc_full[2], acc_empty[2], drain;
+  uint64_t wu_full, acc_full[kPoolAccBufs], acc_empty[kPoolAccBufs], drain;
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -121,7 +124,7 @@ struct PoolTcSmem {
 // kBias: the optional biases inside tanh and sigma (bW, bU) are given; without them (the
 // paper's form) their adds and loads are left out of the per-unit loop.
 template <bool kBias>
-__global__ void __launch_bounds__(kPoolTcThreads, 2)  // two CTAs per SM (TMEM: 2 x 256 columns)
+__global__ void __launch_bounds__(kPoolTcThreads, kPoolCtasPerSm)
     router_pool_tc_kernel(const __grid_constant__ CUtensorMap tmap_q,
                           const __grid_constant__ CUtensorMap tmap_w,
                           const __grid_constant__ CUtensorMap tmap_u, RouterArgs a,
@@ -147,7 +150,7 @@ __global__ void __launch_bounds__(kPoolTcThreads, 2)  // two CTAs per SM (TMEM: 
       mbar_init(&sm.q_empty[s], 128);
     }
     mbar_init(&sm.wu_full, 1);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kPoolAccBufs; ++b) {
       mbar_init(&sm.acc_full[b], 1);
       mbar_init(&sm.acc_empty[b], 128);
     }
@@ -211,9 +214,9 @@ __global__ void __launch_bounds__(kPoolTcThreads, 2)  // two CTAs per SM (TMEM: 
     const uint64_t db = sdesc_sw128(smem_u32(sm.wu));
     bool ok = mbar_wait_warp(&sm.wu_full, 0, err, abort_flag);
     for (int i = 0; i < n_tiles && ok; ++i) {
-      const int st = i % kPoolTcStages, ab = i & 1;
+      const int st = i % kPoolTcStages, ab = i % kPoolAccBufs;
       ok = mbar_wait_warp(&sm.q_full[st], (i / kPoolTcStages) & 1, err, abort_flag) &&
-           mbar_wait_warp(&sm.acc_empty[ab], ((i >> 1) & 1) ^ 1, err, abort_flag);
+           mbar_wait_warp(&sm.acc_empty[ab], ((i / kPoolAccBufs) & 1) ^ 1, err, abort_flag);
       if (!ok) break;
       tc_fence_after();
       const uint64_t da = sdesc_sw128(smem_u32(sm.q[st]));
@@ -238,8 +241,8 @@ __global__ void __launch_bounds__(kPoolTcThreads, 2)  // two CTAs per SM (TMEM: 
     const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
     bool ok = true;
     for (int i = 0; i < n_tiles && ok; ++i) {
-      const int st = i % kPoolTcStages, ab = i & 1;
-      ok = mbar_wait_warp(&sm.acc_full[ab], (i >> 1) & 1, err, abort_flag);
+      const int st = i % kPoolTcStages, ab = i % kPoolAccBufs;
+      ok = mbar_wait_warp(&sm.acc_full[ab], (i / kPoolAccBufs) & 1, err, abort_flag);
       if (!ok) break;
       tc_fence_after();
       float e2x = 0.f, e2y = 0.f;
@@ -645,7 +648,7 @@ cudaError_t launch_router(const RouterArgs& a, const RouterScratch& sc, int num_
   // Pooling sweep on the tensor cores: two CTAs per SM (TMEM 2 x 256 columns), runs of
   // 128-token tiles.
   const int n_tiles = (a.N + 127) / 128;
-  int pool_split = (2 * num_sms + a.H - 1) / a.H;
+  int pool_split = (kPoolCtasPerSm * num_sms + a.H - 1) / a.H;
   pool_split = max(1, min(min(pool_split, kPoolSplitMax), n_tiles));
   CUtensorMap tq, tw, tu;  // Q rows of all heads, W and U as [H 64][64]; 128-byte swizzle
   if ((e = make_tmap_bf16_2d(&tq, a.qkv, (uint64_t)3 * a.H * 64, (uint64_t)a.N,
