@@ -99,9 +99,12 @@ __global__ void merge_setup_kernel(MergeGeo g, const __nv_bfloat16* kbar, __nv_b
 // chunks two CTAs share.
 //   warp 0      TMA: a segment's 128 source rows (16 KB, two buffers) and destination chunks
 //               (256 rows x 64 channels, 32 KB, 128-byte swizzle) through a kMatchStages ring;
-//   warp 1      TMEM owner and MMA issue: four tcgen05.mma M128 N256 K16 per chunk into one
-//               of two 256-column fp32 accumulators (the epilogue of one chunk overlaps the
-//               MMAs of the next);
+//   warp 1      TMEM owner;
+//   warps 1-2   MMA issue: four tcgen05.mma M128 N256 K16 per chunk into one of two 256-column
+//               fp32 accumulators (the epilogue of one chunk overlaps the MMAs of the next),
+//               warp 1 the even chunks (accumulator 0), warp 2 the odd ones: a chunk's waits,
+//               MMA and commit instructions take one warp about 800 clocks, more than the MMAs
+//               themselves (512);
 //   warps 4-19  argmax: a source row (TMEM lane) and a quarter of each chunk's columns per
 //               thread, loaded into registers (two tcgen05.ld.red of 32 columns, which also
 //               return each 32-column piece's maximum) before the accumulator is released; a
@@ -122,7 +125,7 @@ struct MatchSmem {
   float4 stash[kMatchWarps][32][8];  // each argmax thread's best piece, 16-byte slots rotated by lane
   uint64_t src_full[2], src_empty[2];
   uint64_t dst_full[kMatchStages], dst_empty[kMatchStages];
-  uint64_t acc_full[2], acc_empty[2], drain;
+  uint64_t acc_full[2], acc_empty[2], drain[2];
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -168,7 +171,7 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
   if (threadIdx.x == 0) {
     for (int b = 0; b < 2; ++b) {
       mbar_init(&sm.src_full[b], 1);
-      mbar_init(&sm.src_empty[b], 1);
+      mbar_init(&sm.src_empty[b], 2);  // both MMA warps
       mbar_init(&sm.acc_full[b], 1);
       mbar_init(&sm.acc_empty[b], 32 * kMatchWarps);
     }
@@ -176,7 +179,8 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
       mbar_init(&sm.dst_full[s], 1);
       mbar_init(&sm.dst_empty[s], 1);
     }
-    mbar_init(&sm.drain, 1);
+    mbar_init(&sm.drain[0], 1);
+    mbar_init(&sm.drain[1], 1);
     sm.abort_flag = 0;
     fence_mbarrier_init();
     fence_proxy_async_smem();
@@ -233,8 +237,12 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
         }
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------ MMA issue
+    // Warp 1 issues the even chunks, warp 2 the odd ones (ac & 1 picks the accumulator and the
+    // warp); both walk all units so that their counters agree, and both commit the release of
+    // a segment's source tile (its mbarrier counts two).
+    const uint32_t mine = (uint32_t)(warp - 1);
     const uint32_t idesc = idesc_bf16(128, kMatchN, 0, 0);
     uint32_t lc = 0, sc = 0, ac = 0;
     bool ok = true;
@@ -246,6 +254,7 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
       tc_fence_after();
       const uint64_t da = sdesc_sw128(smem_u32(sm.src[sb]));
       for (int ch = sg.c0; ch < sg.c1; ++ch, ++lc, ++ac) {
+        if ((ac & 1) != mine) continue;  // the other warp's chunk
         const int st = lc % kMatchStages;
         const uint32_t ab = ac & 1;
         ok = mbar_wait_warp(&sm.dst_full[st], (lc / kMatchStages) & 1, err, abort_flag) &&
@@ -259,16 +268,18 @@ __global__ void __launch_bounds__(kMatchThreads, 1)
             tc_mma_ss(tmem + ab * kMatchN, da + 2 * kk, db + 2 * kk, idesc, kk > 0 ? 1u : 0u);
           tc_commit(&sm.acc_full[ab]);
           tc_commit(&sm.dst_empty[st]);
-          if (ch == sg.c1 - 1) tc_commit(&sm.src_empty[sb]);
         }
         __syncwarp();
       }
+      if (!ok) break;
+      if (elect_one()) tc_commit(&sm.src_empty[sb]);  // this warp's MMAs on the source tile
+      __syncwarp();
       u += sg.c1 - sg.c0;
     }
     if (!ok) {
       if (elect_one()) {
-        tc_commit(&sm.drain);
-        for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.drain, 0); ++k) {}
+        tc_commit(&sm.drain[mine]);
+        for (int k = 0; k < 1000000 && !mbar_try_wait(&sm.drain[mine], 0); ++k) {}
       }
       __syncwarp();
     }
