@@ -381,12 +381,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue_s = [&](int j) -> bool {
         const uint32_t l = lc0 + j, gg = g0 + j;
         const int st = l % kStages;
-        {  // K landed (lanes 0-15 poll) and S_c read by the softmax (lanes 16-31), at once
+        if constexpr (kParts) {  // K landed (lanes 0-15 poll) and S_c read (lanes 16-31), at once
           const bool hi = lane_id() >= 16;
           if (!__all_sync(0xffffffffu, mbar_wait(hi ? &sm.s_empty[c] : &sm.k_full[st],
                                                  hi ? ((gg & 1) ^ 1) : ((l / kStages) & 1),
                                                  prm.err, abort_flag)))
             return false;
+        } else {
+          if (!mbar_wait_warp(&sm.k_full[st], (l / kStages) & 1, prm.err, abort_flag)) return false;
+          if (!mbar_wait_warp(&sm.s_empty[c], (gg & 1) ^ 1, prm.err, abort_flag)) return false;
         }
         tc_fence_after();
         const uint64_t dk = sdesc_sw128(smem_u32(sm.k[st]));
@@ -408,8 +411,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const uint32_t l = lc0 + j, gg = g0 + j;
         const int st = l % kStages;
-        {  // P_c written (lanes 0-10), V landed (11-21) and, on a unit's first tile, O_c free
-           // (22-31), polled at once: 0.8 % faster in the S = 100 stack than one after another
+        // P_c written, V landed and, on a unit's first tile, O_c free.  The split parts (short
+        // units) poll the three at once in lane groups (0-10, 11-21, 22-31), so that the round
+        // trips overlap; the whole-group instance waits one after another, which measured
+        // 2.6 % faster there (the same parallel polls in both: stack unchanged, all-full layer
+        // slower).
+        if constexpr (kParts) {
           const int grp = lane_id() / 11;
           uint64_t* bar = grp == 0 ? &sm.p_full[c]
                         : grp == 1 ? &sm.v_full[st]
@@ -418,6 +425,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                              : grp == 1 ? ((l / kStages) & 1)
                                         : (j == 0 ? ((ic & 1) ^ 1) : (gg & 1));
           ok = __all_sync(0xffffffffu, mbar_wait(bar, par, prm.err, abort_flag));
+        } else {
+          ok = mbar_wait_warp(&sm.p_full[c], gg & 1, prm.err, abort_flag) &&
+               mbar_wait_warp(&sm.v_full[st], (l / kStages) & 1, prm.err, abort_flag) &&
+               (j > 0 || mbar_wait_warp(&sm.o_empty[c], (ic & 1) ^ 1, prm.err, abort_flag));
         }
         if (!ok) break;
         tc_fence_after();
