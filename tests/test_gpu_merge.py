@@ -225,3 +225,35 @@ def test_one_destination_takes_most_sources(stride):
                                       merge=merge, assign=[got])
     _check_matching(got, infos[0], "one heavy destination")
     compare(_f64(x), want, rel=BF16_STEP, what=f"block with a merged token of {len(src) + 1} members")
+
+
+def test_fewer_tokens_than_a_merge_chunk():
+    """Two views of 14 tokens (5 special, 9 patches), stride 2: 28 tokens, fewer than one
+    32-entry chunk of the merge-means kernel; 4 sources join the 24 destinations."""
+    P, N = 14, 28
+    g = synth.rng(26)
+    w = synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1)
+    x_bits = synth.make_tokens(26, N)
+    force = np.array([[2, 1, 0, 1] * 4])
+    dm = vpb.dims(N, 16)
+    assign = torch.full((N,), -1, dtype=torch.int32, device="cuda")
+    dw = vpb.to_device(w)
+    layers = [vpb.layer_weights(dw, None, vpb.merge_options(2, P, 5, assign))]
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK_MERGE)
+    x = vpb.bf16_from_bits(x_bits)
+    modes = torch.zeros(1, 16, dtype=torch.int32, device="cuda")
+    s = torch.zeros(1, 16, device="cuda")
+    vpb.vp_global_stack(dm, x, layers, torch.tensor(force, dtype=torch.int32, device="cuda"), modes, s, 1e-6, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    got = assign.cpu().numpy().astype(np.int64)
+    row_of, dst_tok = oracle.destinations(N, P, 5, 2)
+    assert len(dst_tok) == 24 and int((row_of < 0).sum()) == 4
+    assert np.array_equal(got[row_of >= 0], row_of[row_of >= 0])
+    merge = [{"stride": 2, "tokens_per_view": P, "patch_start": 5}]
+    want, infos = oracle.global_stack(oracle.bf16_bits_to_f64(x_bits), [oracle.load_layer(w)], force_modes=force,
+                                      merge=merge, assign=[got])
+    sc = infos[0]["merge"]["scores"]
+    src = np.nonzero(row_of < 0)[0]
+    assert np.all(sc[src, got[src]] >= sc[src].max(axis=1) - 2e-2)  # each source at a best destination
+    compare(_f64(x), want, rel=BF16_STEP, what="28-token block with merging")
