@@ -242,7 +242,10 @@ __global__ void __launch_bounds__(kPoolTcThreads, kPoolCtasPerSm)
     bool ok = true;
     for (int i = 0; i < n_tiles && ok; ++i) {
       const int st = i % kPoolTcStages, ab = i % kPoolAccBufs;
-      ok = mbar_wait_warp(&sm.acc_full[ab], (i / kPoolAccBufs) & 1, err, abort_flag);
+      // The tile's accumulator, and its Q rows in shared memory (read below by these threads:
+      // they wait on the TMA's barrier themselves rather than rely on the MMA's).
+      ok = mbar_wait_warp(&sm.acc_full[ab], (i / kPoolAccBufs) & 1, err, abort_flag) &&
+           mbar_wait_warp(&sm.q_full[st], (i / kPoolTcStages) & 1, err, abort_flag);
       if (!ok) break;
       tc_fence_after();
       float e2x = 0.f, e2y = 0.f;
@@ -296,6 +299,11 @@ __global__ void __launch_bounds__(kPoolTcThreads, kPoolCtasPerSm)
           }
         }
       }
+      // The stage goes back to the TMA producer: the generic-proxy reads of the Q row above
+      // are ordered before the async-proxy writes that refill it.  Without the fence the release
+      // can overtake loads still in flight: a version with a two-stage ring gave q_pool values
+      // up to 3 % off in repeated runs.
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_arrive(&sm.q_empty[st]);
     }
   }
