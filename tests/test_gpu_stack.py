@@ -109,6 +109,24 @@ def test_stack_three_blocks_all_modes():
                 assert got_s == 0.0, (l, h, got_s)
 
 
+def test_stack_repeated_runs_are_bit_identical():
+    """Two runs of a 3-block stack at 6,000 tokens (every route, several tiles per pooling CTA)
+    on the same tokens give the same bits: every reduction in the library has a fixed order
+    (token merging is not part of this, since a merged token sums its members in fill order)."""
+    N, L = 6000, 3
+    g = synth.rng(7)
+    wts = [synth.make_layer_weights(g, block=True, bias_std=0.05, norm_jitter=0.1) for _ in range(L)]
+    x_bits = synth.make_tokens(7, N)
+    force = np.array([synth.forced_mix(16, f) for f in (0.25, 0.5, 1.0)])
+    a, ma, sa = _run_stack(x_bits, wts, N, force)
+    sat_a = _run_stack.s_attn.copy()
+    b, mb, sb = _run_stack(x_bits, wts, N, force)
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_array_equal(ma, mb)
+    np.testing.assert_array_equal(sa, sb)
+    np.testing.assert_array_equal(sat_a, _run_stack.s_attn)
+
+
 def test_stack_24_blocks_s4_natural_routing():
     """24 blocks over S=4 views at 224 px (1,044 tokens): untrained routers route every
     head of every block to mean (saliency ~ 1/N)."""
