@@ -383,6 +383,8 @@ def run_ours(args):
         line["qkv_positional"] = qk_probe(vpb, dev, N, dws[0])
     if args.tome:
         line["token_merging_s100"] = tome_probe(vpb, dev, N, dws, fm)
+    if args.full_stack:
+        line["all_full_stack_s100"] = all_full_stack_probe(vpb, dev, N, dws, line)
     if args.mix:
         line["mix_sweep_s64"] = mix_probe(vpb, dev, pk)
     if args.saliency:
@@ -502,6 +504,45 @@ def tome_probe(vpb, dev, N, dws, fm, steps=3, warmup=2):
         out[f"stride_{stride}"] = {"merged_fraction": 1 - n_rows / N, "merged_tokens": n_rows,
                                    "ms_per_forward": t, "views_per_s": WORKLOAD.views / t * 1e3,
                                    "kernels_ms": {k: v / steps for k, v in ms.items() if cnt[k]}}
+    return out
+
+
+def all_full_stack_probe(vpb, dev, N, dws, line, steps=2, warmup=1):
+    """The same S = 100 stack with every head of every block forced to full softmax attention
+    (the stack without routing, VGGT's global attention), same weights and tokens; and the
+    routed stack's speedups over it, with and without token merging (the paper's 8x and
+    11x / 14x figures are end-to-end model times on other hardware: context only)."""
+    import torch
+    L = len(dws)
+    x0 = vpb.bf16_from_bits(synth.make_tokens(WORKLOAD.seed, N), dev)
+    x = torch.empty_like(x0)
+    dm = vpb.dims(N, H)
+    ws = vpb.workspace(dm, vpb.VP_WS_STACK, dev)
+    layers = [vpb.layer_weights(w) for w in dws]
+    fm = torch.full((L, H), synth.MODE_FULL, dtype=torch.int32, device=dev)
+    modes = torch.zeros(L, H, dtype=torch.int32, device=dev)
+    s = torch.zeros(L, H, device=dev)
+
+    def step():
+        x.copy_(x0)
+        vpb.vp_global_stack(dm, x, layers, fm, modes, s, 1e-6, ws)
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    t = a.elapsed_time(b) / steps
+    full_vps = WORKLOAD.views / t * 1e3
+    out = {"ms_per_forward": t, "views_per_s": full_vps, "full_heads": L * H, "steps": steps,
+           "speedup_routed": line["value"] / full_vps}
+    tome = line.get("token_merging_s100")
+    if tome:
+        for k, v in tome.items():
+            out[f"speedup_routed_and_merged_{k}"] = v["views_per_s"] / full_vps
     return out
 
 
@@ -825,6 +866,8 @@ def main():
     ap.add_argument("--no-qk", dest="qk", action="store_false")
     ap.add_argument("--no-tome", dest="tome", action="store_false")
     ap.add_argument("--no-mix", dest="mix", action="store_false", help="skip the S=64 routing-mix sweep")
+    ap.add_argument("--no-full-stack", dest="full_stack", action="store_false",
+                    help="skip the S=100 stack with every head full (about 3 s of GPU time)")
     ap.add_argument("--no-saliency", dest="saliency", action="store_false",
                     help="skip the router-vs-exact saliency report")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
