@@ -305,8 +305,9 @@ vp_status vp_global_stack(const vp_dims* dims, int32_t n_layers, vp_bf16* x_inou
  * writes the host memory through its device-visible address, so x_in and x_out must be
  * page-locked (cudaHostAlloc, cudaHostRegister, or a framework's pinned allocator): other
  * host memory returns VP_ERR_INVALID_ARG.  Everything is enqueued on `stream` and the call
- * returns without waiting; x_out is complete once the stream is.  The other arguments are
- * those of vp_global_stack.  All pointers 16-byte aligned.
+ * returns without waiting: x_in is read, and x_out written, while the stream runs, so the caller
+ * leaves both untouched (and allocated) until the stream has completed; x_out is then complete.
+ * The other arguments are those of vp_global_stack.  All pointers 16-byte aligned.
  */
 vp_status vp_global_stack_host(const vp_dims* dims, int32_t n_layers, const vp_bf16* x_in,
                                vp_bf16* x_out, vp_bf16* x_dev, const vp_layer_weights* layers,
