@@ -134,6 +134,9 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
 // Surrogate (§4.3, the method's form and the mean-context ablation) and mean heads on the
 // tensor cores, queued behind the full-attention kernel (heads_cheap_tc.cu).
 cudaError_t launch_cheap_heads_tc(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+// §5 linear-attention state of every surrogate head into a.lin_state (zeroed by the caller),
+// on the tensor cores (linear_state_tc.cu).
+cudaError_t launch_linear_state_tc(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
 // All heads of a layer: full-mode heads, then surrogate and mean heads overlapped with the
 // full-attention tail (heads_cheap.cu).
 cudaError_t launch_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
