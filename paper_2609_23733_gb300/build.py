@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libvp.so")
 SOURCES = ["api.cu", "router.cu", "attn_full.cu", "heads_cheap.cu", "heads_cheap_tc.cu", "gemm.cu",
-           "layernorm.cu", "router_noalloc.cu", "merge.cu", "host_copy.cu", "linear_state_tc.cu"]
+           "layernorm.cu", "router_noalloc.cu", "merge.cu", "host_copy.cu", "linear_attn_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

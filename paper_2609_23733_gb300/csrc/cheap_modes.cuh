@@ -74,91 +74,6 @@ __device__ __forceinline__ void mean_item(const HeadAttnArgs& a, int h, int chun
   broadcast_rows(a, a.mean_v + h * 64, h, chunk * kMeanRows, kMeanRows, tid);
 }
 
-// ---------------------------------------------------------------- §5 linear attention
-// phi(x) = elu(x) + 1 (Katharopoulos et al. 2020), in fp32.
-__device__ __forceinline__ float elu1(float x) { return x > 0.f ? x + 1.f : __expf(x); }
-
-struct LinSmem {
-  // S_h^T [e][c] as bf16 hi + lo parts (hi = bf16(S), lo = bf16(S - hi): 16 significant
-  // bits), padded rows like the surrogate's weights; z_h in fp32.
-  __nv_bfloat16 st_hi[64 * kBStride];
-  __nv_bfloat16 st_lo[64 * kBStride];
-  float z[64];
-};
-
-__device__ __forceinline__ void linear_stage(const HeadAttnArgs& a, LinSmem& sm, int h, int tid) {
-  const float* src = a.lin_state + (size_t)h * kLinState;
-  for (int i = tid; i < 64 * 64; i += 256) {
-    const int c = i >> 6, e = i & 63;  // coalesced over e
-    const float v = __ldcg(src + i);
-    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-    sm.st_hi[e * kBStride + c] = hi;
-    sm.st_lo[e * kBStride + c] = __float2bfloat16_rn(v - __bfloat162float(hi));
-  }
-  if (tid < 64) sm.z[tid] = __ldcg(src + 64 * 64 + tid);
-}
-
-// Surrogate head h in linear-attention form, 16 rows [chunk * 128 + 16 w, +16) for warp w:
-// y_i = phi(q_i)^T S_h / phi(q_i)^T z_h.  The numerator runs on the tensor cores (mma.sync,
-// phi(Q) rounded to bf16, S_h as hi + lo bf16 parts, fp32 accumulation) with the same
-// permuted reduction index as surrogate_rows; the denominator in fp32 from the same rows.
-// Not inlined: its registers then do not add to those of the kernel's other paths.
-static __device__ __noinline__ void linear_rows(const HeadAttnArgs& a, const LinSmem& sm, int h,
-                                            int chunk, int w, int lane) {
-  const int N = a.N, H = a.H;
-  const size_t row_pitch = (size_t)3 * H * kHeadDim;
-  const int r = lane >> 2, c = lane & 3;
-  const int base = chunk * kSurrRows + w * 16;
-  if (base >= N) return;
-  const int ra = base + r, rb = base + r + 8;
-  const bool va = ra < N, vb = rb < N;
-  uint32_t qa[8], qb[8];
-  float da = 0.f, db = 0.f;
-  {
-    const __nv_bfloat16* qbase = a.qkv + (size_t)h * kHeadDim + 16 * c;
-    const uint4* pa = reinterpret_cast<const uint4*>(qbase + (size_t)(va ? ra : base) * row_pitch);
-    const uint4* pb = reinterpret_cast<const uint4*>(qbase + (size_t)(vb ? rb : base) * row_pitch);
-    const uint4 x0 = __ldg(pa), x1 = __ldg(pa + 1), y0 = __ldg(pb), y1 = __ldg(pb + 1);
-    const uint32_t xa[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-    const uint32_t xb[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
-#pragma unroll
-    for (int m = 0; m < 8; ++m) {  // word m holds channels 16c + 2m, 16c + 2m + 1
-      const float a0 = elu1(bf16_lo(xa[m])), a1 = elu1(bf16_hi(xa[m]));
-      const float b0 = elu1(bf16_lo(xb[m])), b1 = elu1(bf16_hi(xb[m]));
-      const float z0 = sm.z[16 * c + 2 * m], z1 = sm.z[16 * c + 2 * m + 1];
-      da = fmaf(a0, z0, fmaf(a1, z1, da));
-      db = fmaf(b0, z0, fmaf(b1, z1, db));
-      qa[m] = pack_bf16x2(a0, a1);
-      qb[m] = pack_bf16x2(b0, b1);
-    }
-  }
-  da += __shfl_xor_sync(0xffffffffu, da, 1);
-  da += __shfl_xor_sync(0xffffffffu, da, 2);
-  db += __shfl_xor_sync(0xffffffffu, db, 1);
-  db += __shfl_xor_sync(0xffffffffu, db, 2);
-  const float ia = 1.f / da, ib = 1.f / db;
-  __nv_bfloat16* ya = a.y + ((size_t)ra * H + h) * 64;
-  __nv_bfloat16* yb = a.y + ((size_t)rb * H + h) * 64;
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {  // output channels 8j .. 8j + 7
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    const uint4* ph = reinterpret_cast<const uint4*>(&sm.st_hi[(8 * j + r) * kBStride + 16 * c]);
-    const uint4* pl = reinterpret_cast<const uint4*>(&sm.st_lo[(8 * j + r) * kBStride + 16 * c]);
-    const uint4 h0 = ph[0], h1 = ph[1], l0 = pl[0], l1 = pl[1];
-    const uint32_t bh[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
-    const uint32_t bl[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      const uint32_t af[4] = {qa[2 * kk], qb[2 * kk], qa[2 * kk + 1], qb[2 * kk + 1]};
-      mma_bf16_16816(acc, af, bh[2 * kk], bh[2 * kk + 1]);
-      mma_bf16_16816(acc, af, bl[2 * kk], bl[2 * kk + 1]);
-    }
-    const int col = 8 * j + 2 * c;
-    if (va) *reinterpret_cast<uint32_t*>(ya + col) = pack_bf16x2(acc[0] * ia, acc[1] * ia);
-    if (vb) *reinterpret_cast<uint32_t*>(yb + col) = pack_bf16x2(acc[2] * ib, acc[3] * ib);
-  }
-}
-
 // Stages head h's surrogate weights (both MLPs' value halves of layer 1, both layer 2s,
 // biases and C_h).  The context half of layer 1 is folded into c1 by surrogate_fold after
 // the group has synchronised.

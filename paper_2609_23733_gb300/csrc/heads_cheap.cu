@@ -18,11 +18,7 @@ namespace {
 constexpr int kThreads = 256;
 
 __global__ void __launch_bounds__(kThreads, 3) cheap_heads_kernel(HeadAttnArgs a) {
-  __shared__ __align__(16) union {
-    cheap::SurrSmem surr;
-    cheap::LinSmem lin;
-  } sm;
-  cheap::SurrSmem& surr = sm.surr;
+  __shared__ __align__(16) cheap::SurrSmem surr;
   __shared__ int s_item;
   const int tid = threadIdx.x, lane = tid & 31;
   const int s_first = __ldg(a.offsets + 1), m_first = __ldg(a.offsets + 0);
@@ -30,7 +26,9 @@ __global__ void __launch_bounds__(kThreads, 3) cheap_heads_kernel(HeadAttnArgs a
   const int n_mean = s_first - m_first;
   const int s_chunks = (a.N + cheap::kSurrRows - 1) / cheap::kSurrRows;
   const int m_chunks = (a.N + cheap::kMeanRows - 1) / cheap::kMeanRows;
-  const int items = n_surr * s_chunks + n_mean * m_chunks;
+  // The linear-attention form of the surrogate heads runs in its own kernels, before this one.
+  const int s_items = (a.variant & VP_VARIANT_LINEAR_ATTENTION) ? 0 : n_surr * s_chunks;
+  const int items = s_items + n_mean * m_chunks;
   int cur_h = -1;
   // Items in order: surrogate rows (head-major), then mean rows; taken from a counter so
   // that CTAs started early (on SMs freed early) do more of them.
@@ -40,20 +38,11 @@ __global__ void __launch_bounds__(kThreads, 3) cheap_heads_kernel(HeadAttnArgs a
     __syncthreads();
     const int it = s_item;
     if (it >= items) break;
-    if (it < n_surr * s_chunks) {
+    if (it < s_items) {
       const int slot = it / s_chunks, chunk = it - slot * s_chunks;
       const int h = __ldg(a.head_ids + s_first + slot);
       if (a.variant & VP_VARIANT_NO_RESIDUAL) {  // §5: y_i = C_h, no token-wise correction
         cheap::broadcast_rows(a, a.ctx + h * 64, h, chunk * cheap::kSurrRows, cheap::kSurrRows, tid);
-        continue;
-      }
-      if (a.variant & VP_VARIANT_LINEAR_ATTENTION) {  // §5: linear attention instead
-        if (h != cur_h) {
-          cheap::linear_stage(a, sm.lin, h, tid);
-          __syncthreads();
-          cur_h = h;
-        }
-        cheap::linear_rows(a, sm.lin, h, chunk, tid >> 5, lane);
         continue;
       }
       if (h != cur_h) {
@@ -65,7 +54,7 @@ __global__ void __launch_bounds__(kThreads, 3) cheap_heads_kernel(HeadAttnArgs a
       }
       cheap::surrogate_rows(a, surr, h, chunk, tid >> 5, lane);
     } else {
-      const int it2 = it - n_surr * s_chunks;
+      const int it2 = it - s_items;
       const int slot = it2 / m_chunks, chunk = it2 - slot * m_chunks;
       cheap::mean_item(a, __ldg(a.head_ids + m_first + slot), chunk, tid);
     }
@@ -86,12 +75,14 @@ cudaError_t launch_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st) {
     if (e != cudaSuccess) return e;
   }
   if (a.variant & VP_VARIANT_LINEAR_ATTENTION) {
-    // The state is complete before the full-attention kernel starts, hence before the
-    // cheap-heads kernel (which follows that one) reads it.
+    // The surrogate heads in linear-attention form, state then apply, before the
+    // full-attention kernel; the mean heads stay in the cheap-heads kernel behind it.
     e = cudaMemsetAsync(a.lin_state, 0, sizeof(float) * kLinState * a.H, st);
     if (e != cudaSuccess) return e;
     prof_before(VP_KERNEL_SURROGATE, st);
     e = launch_linear_state_tc(a, num_sms, st);
+    if (e == cudaSuccess) e = launch_linear_apply_tc(a, num_sms, st);
+    prof_extra_launch();
     prof_after(st);
     if (e != cudaSuccess) return e;
   }

@@ -135,8 +135,11 @@ cudaError_t launch_full_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t s
 // tensor cores, queued behind the full-attention kernel (heads_cheap_tc.cu).
 cudaError_t launch_cheap_heads_tc(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
 // §5 linear-attention state of every surrogate head into a.lin_state (zeroed by the caller),
-// on the tensor cores (linear_state_tc.cu).
+// on the tensor cores (linear_attn_tc.cu).
 cudaError_t launch_linear_state_tc(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
+// §5 linear-attention output of every surrogate head from that state, y_i = phi(q_i)^T S /
+// phi(q_i)^T z, on the tensor cores (linear_attn_tc.cu).
+cudaError_t launch_linear_apply_tc(const HeadAttnArgs& a, int num_sms, cudaStream_t st);
 // All heads of a layer: full-mode heads, then surrogate and mean heads overlapped with the
 // full-attention tail (heads_cheap.cu).
 cudaError_t launch_heads(const HeadAttnArgs& a, int num_sms, cudaStream_t st);

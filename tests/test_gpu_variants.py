@@ -127,6 +127,42 @@ def test_linear_attention_heads(N):
     compare(got[:, 3], oracle.round_bf16(np.tile(q[:, 2, 3].mean(0), (N, 1))), what="mean")
 
 
+@pytest.mark.parametrize("N,H", [(50_000, 4), (137_400, 16)])
+def test_linear_attention_heads_sampled_rows(N, H):
+    """The linear-attention variant at sizes where every CTA of both kernels takes several
+    token tiles (the 16-head, 137,400-token case is the S = 100 stack's head geometry): sampled
+    rows of every linear head against the oracle's definition, and the mean head in full."""
+    g = np.random.default_rng(N + H)
+    # Standard normal x 1.5, drawn in bf16 by torch's seeded CPU generator (numpy's float32
+    # draw and rounding take minutes at 422 M values).
+    x = torch.randn(N, 3 * H * 64, generator=torch.Generator().manual_seed(N + H)) * 1.5
+    bits = x.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16).reshape(N, 3, H, 64)
+    del x
+    modes = np.ones(H, np.int32)
+    modes[H - 1] = 0
+    ids_o, off_o, _ = oracle.bin_heads(modes, N)
+    dm = vpb.dims(N, H, variant=FLAG["linear_attention"])
+    w = vpb.to_device(synth.make_layer_weights(synth.rng(1), D=H * 64, H=H))
+    ws = vpb.workspace(dm, vpb.VP_WS_ROUTER)
+    y = torch.full((N, H * 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+    v_last = oracle.bf16_bits_to_f64(bits[:, 2, H - 1])
+    mv = torch.zeros(H, 64, dtype=torch.float32, device="cuda")
+    mv[H - 1] = torch.tensor(v_last.mean(0), dtype=torch.float32)
+    vpb.vp_head_attention(dm, vpb.bf16_from_bits(bits.reshape(N, -1)), torch.tensor(ids_o, device="cuda"),
+                          torch.tensor(off_o, device="cuda"), torch.zeros(H, 64, device="cuda"), mv,
+                          vpb.surrogate_weights(w), y, ws)
+    torch.cuda.synchronize()
+    assert vpb.vp_read_device_error(ws) == 0
+    got = y.float().cpu().numpy().reshape(N, H, 64)
+    edges = [0, 1, 127, 128, 129, N // 2, N - 129, N - 128, N - 1]
+    for h in range(H - 1):
+        rows = np.unique(np.concatenate([edges, g.choice(N, 192, replace=False)]))
+        q, k, v = (oracle.bf16_bits_to_f64(bits[:, j, h]) for j in range(3))
+        want = oracle.linear_attention(q, k, v, rows=rows)
+        compare(got[rows, h], oracle.round_bf16(want), what=f"linear head {h}")
+    compare(got[:, H - 1], oracle.round_bf16(np.tile(v_last.mean(0), (N, 1))), what="mean")
+
+
 def test_variant_validation():
     import ctypes
     lib = vpb.lib()
