@@ -769,9 +769,10 @@ def kernel_case(args):
     dev = torch.device("cuda:0")
     N = args.case_tokens
     qkv = torch.randn(N, 3 * D, device=dev).to(torch.bfloat16)
-    if args.kernel_case in ("layer_norm", "router", "surrogate", "mean"):
+    if args.kernel_case in ("layer_norm", "router", "surrogate", "mean", "linear"):
         w = vpb.to_device(synth.make_layer_weights(synth.rng(0), block=True), dev)
-        dm = vpb.dims(N, H)
+        # linear: every head a surrogate head in the section-5 linear-attention form
+        dm = vpb.dims(N, H, variant=vpb.VP_VARIANT_LINEAR_ATTENTION if args.kernel_case == "linear" else 0)
         ws = vpb.workspace(dm, vpb.VP_WS_ROUTER, dev)
         x = torch.randn(N, D, device=dev).to(torch.bfloat16)
         y = torch.empty(N, D, dtype=torch.bfloat16, device=dev)
@@ -886,7 +887,7 @@ def main():
     ap.add_argument("--no-saliency", dest="saliency", action="store_false",
                     help="skip the router-vs-exact saliency report")
     ap.add_argument("--kernel-case", choices=["attn_full", "gemm", "gemm_fc1", "gemm_wo", "layer_norm", "router",
-                                              "surrogate", "mean", "bin", "merge"],
+                                              "surrogate", "mean", "linear", "bin", "merge"],
                     default=None,
                     help="run one kernel on a mid-sized input (for ncu captures) and exit")
     ap.add_argument("--case-tokens", type=int, default=32768)

@@ -38,7 +38,6 @@
 // Every wait is bounded (mbar_wait); on timeout the CTA records VP_DEVERR_WAIT_TIMEOUT, stops,
 // waits (bounded) for its own copies and MMAs, frees TMEM and exits.  The groups agree on
 // stopping through reduction barriers, so that no thread is left at a named barrier.
-#include "cheap_modes.cuh"
 #include "common.cuh"
 #include "internal.h"
 
