@@ -308,10 +308,12 @@ SurrogateArgs make_surrogate_args(const vp_surrogate_weights* sw) {
 }
 
 // Runs the three mode kernels for bins already in device memory.
+// skip_mean_y: the mean heads' rows of Y are left unwritten (their part of W_O is folded into
+// its bias, launch_wo_mean_fold).
 vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* head_ids,
                     const int32_t* offsets, const float* ctx, const float* mean_v,
                     const vp_surrogate_weights* sw, __nv_bfloat16* y, float* s_attn,
-                    const RouterScratch& sc, cudaStream_t st) {
+                    const RouterScratch& sc, cudaStream_t st, bool skip_mean_y = false) {
   HeadAttnArgs ha{};
   ha.N = dm->N;
   ha.H = dm->H;
@@ -331,10 +333,15 @@ vp_status run_heads(const vp_dims* dm, const __nv_bfloat16* qkv, const int32_t* 
   ha.s_attn = s_attn;
   ha.err = sc.err;
   ha.cheap_counter = sc.cheap_counter;
+  ha.skip_mean_y = skip_mean_y ? 1 : 0;
   return from_cuda(launch_heads(ha, device_sm_count(), st));
 }
 
 // QKV projection -> router -> bins -> heads -> W_O (+ optional LayerScale / residual).
+// A mean head's rows of Y are all mu_h = bf16(mean of V_h), so its part of Y W_O^T is the
+// same vector for every token: it goes into W_O's bias (launch_wo_mean_fold) and the W_O GEMM
+// leaves that head's 64 K columns out; its rows of Y are written only when the caller asked
+// for Y (keep_mean_y).
 // LayerNorm folded into a layer's QKV projection: xin is then the raw residual stream and
 // w_qkv / b_qkv the folded weights (see LinearArgs).
 struct LnFold {
@@ -349,7 +356,8 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
                     const vp_surrogate_weights* sw, const int32_t* force_modes,
                     __nv_bfloat16* out, __nv_bfloat16* qkv, __nv_bfloat16* y, float* s_out,
                     float* s_attn_out, int32_t* modes_out, const RouterScratch& sc,
-                    cudaStream_t st, const LnFold* fold = nullptr, const QkArgs* qk = nullptr) {
+                    cudaStream_t st, const LnFold* fold = nullptr, const QkArgs* qk = nullptr,
+                    bool keep_mean_y = false) {
   const int N = dm->N, D = dm->H * kHeadDim;
   const int sms = device_sm_count();
   LinearArgs la{};
@@ -373,15 +381,22 @@ vp_status run_layer(const vp_dims* dm, const __nv_bfloat16* xin, const vp_bf16* 
   ra.s_out = s_out;
   ra.modes_out = modes_out;
   VP_TRY(from_cuda(launch_router(ra, sc, sms, st)));
+  prof_before(VP_KERNEL_GEMM, st);  // W_O's bias, counted with the projections
+  const cudaError_t ef = launch_wo_mean_fold(D, dm->H, reinterpret_cast<const __nv_bfloat16*>(w_o),
+                                             b_o, sc.mean_v, sc.head_ids, sc.offsets, sc.wo_bias, st);
+  prof_after(st);
+  VP_TRY(from_cuda(ef));
   VP_TRY(run_heads(dm, qkv, sc.head_ids, sc.offsets, sc.ctx, sc.mean_v, sw, y, s_attn_out, sc,
-                   st));
+                   st, !keep_mean_y));
   LinearArgs lo{};
   lo.M = N;
   lo.N = D;
   lo.K = D;
   lo.A = y;
   lo.W = reinterpret_cast<const __nv_bfloat16*>(w_o);
-  lo.bias = b_o;
+  lo.bias = sc.wo_bias;  // b_O + the mean heads' rows of Y times W_O
+  lo.skip_ids = sc.head_ids;  // the mean heads' K columns left out
+  lo.skip_off = sc.offsets;
   lo.act = VP_ACT_NONE;
   lo.scale = ls1;
   lo.residual = residual;
@@ -613,7 +628,7 @@ vp_status vp_moh_global_attention(const vp_dims* dims, const vp_bf16* x, const v
   if (y_out) y = reinterpret_cast<__nv_bfloat16*>(y_out);
   return run_layer(dims, reinterpret_cast<const __nv_bfloat16*>(x), w_qkv, b_qkv, w_o, b_o,
                    nullptr, nullptr, rw, sw, force_modes, reinterpret_cast<__nv_bfloat16*>(out),
-                   qkv, y, s_out, s_attn_out, modes_out, sc, st, nullptr, &qa);
+                   qkv, y, s_out, s_attn_out, modes_out, sc, st, nullptr, &qa, y_out != nullptr);
 }
 
 // The host-side checks of vp_global_stack (also run by vp_global_stack_host before it

@@ -34,6 +34,7 @@ struct GemmSmem {
   uint64_t full[kStages], empty[kStages];
   uint64_t acc_full[2], acc_empty[2], drain;
   uint32_t tmem_base;
+  uint32_t skip_mask;  // K-blocks left out (LinearArgs::skip_ids)
   int abort_flag;
 };
 
@@ -58,6 +59,8 @@ struct GemmParams {
   const float2* rope_cs;
   int tok_per_view, patch_start, grid_w;
   const int32_t* tok_index;
+  const int32_t* skip_ids;
+  const int32_t* skip_off;
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -86,6 +89,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&sm.drain, 1);
     sm.abort_flag = 0;
+    uint32_t skip = 0;
+    if (prm.skip_ids) {
+      const int s0 = __ldg(prm.skip_off), s1 = __ldg(prm.skip_off + 1);
+      for (int i = s0; i < s1; ++i) skip |= 1u << (__ldg(prm.skip_ids + i) & 31);
+    }
+    sm.skip_mask = skip;
     fence_mbarrier_init();
     fence_proxy_async_smem();
     tma_prefetch_desc(&tmap_a);
@@ -100,6 +109,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
+  // K-blocks left out, and whether that is all of them (the accumulator is then 0).
+  const uint32_t skip = sm.skip_mask;
+  const bool acc_zero = skip != 0 && __popc(skip & (k_blocks >= 32 ? 0xffffffffu : (1u << k_blocks) - 1u)) == k_blocks;
 
   if (warp == 0) {
     // TMA producer: converged warp (warp-uniform coordinates), one elected lane issues.
@@ -107,7 +119,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
       const int mt = t / n_tiles, nt = t - mt * n_tiles;
-      for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
+      for (int kb = 0; kb < k_blocks; ++kb) {
+        if ((skip >> kb) & 1u) continue;
         const int st = lc % kStages;
         ok = mbar_wait_warp(&sm.empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
         if (!ok) break;
@@ -117,6 +130,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(sm.b[st], &tmap_b, &sm.full[st], kb * kBK, nt * kBN);
         }
         __syncwarp();
+        ++lc;
       }
     }
     if (!ok && lane == 0) {
@@ -139,7 +153,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t d = tmem + ab * kBN;
-      for (int kb = 0; kb < k_blocks; ++kb, ++lc) {
+      bool first = true;  // the tile's first MMA overwrites the accumulator
+      for (int kb = 0; kb < k_blocks; ++kb) {
+        if ((skip >> kb) & 1u) continue;
         const int st = lc % kStages;
         ok = mbar_wait_warp(&sm.full[st], (lc / kStages) & 1, prm.err, abort_flag);
         if (!ok) break;
@@ -149,10 +165,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
-            tc_mma_ss(d, da + 2 * kk, db + 2 * kk, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+            tc_mma_ss(d, da + 2 * kk, db + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
           tc_commit(&sm.empty[st]);
         }
         __syncwarp();
+        first = false;
+        ++lc;
       }
       if (!ok) break;
       if (elect_one()) tc_commit(&sm.acc_full[ab]);
@@ -378,6 +396,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int cc = 0; cc < 4; ++cc) {
         if (cc + 1 < 4) tmem_ld32(tcol + 32 * (cc + 1), v[(cc + 1) & 1]);  // in flight meanwhile
         float* x = v[cc & 1];
+        if (acc_zero) {  // every K-block left out: A W^T is 0 (TMEM was not written)
+#pragma unroll
+          for (int k = 0; k < 32; ++k) x[k] = 0.f;
+        }
         const int col0 = nt * kBN + half * 128 + cc * 32;
         if (col0 < N) {
           // Bias, GELU, LayerScale and residual on column pairs (packed f32x2 arithmetic).
@@ -476,9 +498,44 @@ __global__ void rope_table_kernel(int max_pos, double base, float2* table) {
 
 }  // namespace
 
+namespace {
+
+// A warp per output column n of W_O: lane l takes channels 2 l, 2 l + 1 of every mean head.
+__global__ void wo_mean_fold_kernel(int D, int H, const __nv_bfloat16* w_o, const float* b_o,
+                                    const float* mean_v, const int32_t* head_ids,
+                                    const int32_t* offsets, float* bias_out) {
+  const int n = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+  if (n >= D) return;  // whole warps
+  const int m0 = __ldg(offsets), m1 = __ldg(offsets + 1);
+  const __nv_bfloat16* wrow = w_o + (size_t)n * H * 64 + 2 * lane;
+  float acc = 0.f;
+  for (int i = m0; i < m1; ++i) {
+    const int h = __ldg(head_ids + i);
+    const uint32_t w2 = __ldg(reinterpret_cast<const unsigned int*>(wrow + h * 64));
+    // the mean head's row of Y as stored: bf16(mean_v), round to nearest even
+    const float2 mv = __ldg(reinterpret_cast<const float2*>(mean_v + h * 64) + lane);
+    const uint32_t mu = pack_bf16x2(mv.x, mv.y);
+    acc = fmaf(bf16_lo(mu), bf16_lo(w2), fmaf(bf16_hi(mu), bf16_hi(w2), acc));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) bias_out[n] = (b_o ? __ldg(b_o + n) : 0.f) + acc;
+}
+
+}  // namespace
+
 cudaError_t launch_rope_table(int max_pos, float base, float2* table, cudaStream_t st) {
   const int n = (max_pos + 1) * 16;
   rope_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(max_pos, (double)base, table);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wo_mean_fold(int D, int H, const __nv_bfloat16* w_o, const float* b_o,
+                                const float* mean_v, const int32_t* head_ids,
+                                const int32_t* offsets, float* bias_out, cudaStream_t st) {
+  const int threads = 256, blocks = (D * 32 + threads - 1) / threads;
+  wo_mean_fold_kernel<<<blocks, threads, 0, st>>>(D, H, w_o, b_o, mean_v, head_ids, offsets,
+                                                  bias_out);
   return cudaGetLastError();
 }
 
@@ -498,6 +555,8 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
       (a.part_out && a.N % 128 != 0))
     return cudaErrorInvalidValue;
   const bool qk = a.qk_cols > 0;
+  if (a.skip_ids && (!a.skip_off || a.ln_part || qk || a.K % kBK != 0 || a.K > 32 * kBK))
+    return cudaErrorInvalidValue;
   if (qk && (a.qk_cols % 256 != 0 || a.qk_cols > a.N || a.act != VP_ACT_NONE || a.scale ||
              a.residual || a.part_out || (!a.qn_g != !a.qn_b) || (!a.kn_g != !a.kn_b) ||
              (a.rope_cs && (a.tok_per_view < 1 || a.grid_w < 1 || a.patch_start < 0))))
@@ -505,7 +564,7 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   GemmParams prm{a.M,     a.N,   a.K,   a.bias,      a.act,  a.scale,   a.residual,
                  a.out,   a.err, a.ln_part, a.ln_c, a.ln_eps, a.part_out,
                  qk ? a.qk_cols : 0, a.qn_g, a.qn_b, a.kn_g, a.kn_b, a.qk_eps, a.rope_cs,
-                 a.tok_per_view, a.patch_start, a.grid_w, a.tok_index};
+                 a.tok_per_view, a.patch_start, a.grid_w, a.tok_index, a.skip_ids, a.skip_off};
   prof_before(VP_KERNEL_GEMM, st);
   gemm_kernel<<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
   prof_after(st);

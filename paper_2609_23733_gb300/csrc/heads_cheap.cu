@@ -46,7 +46,7 @@ __global__ void __launch_bounds__(kThreads, 3) broadcast_heads_kernel(HeadAttnAr
   const int chunks = (a.N + kRows - 1) / kRows;
   // Surrogate heads are broadcast rows only without the token-wise correction.
   const int s_items = (a.variant & VP_VARIANT_NO_RESIDUAL) ? n_surr * chunks : 0;
-  const int items = s_items + n_mean * chunks;
+  const int items = s_items + (a.skip_mean_y ? 0 : n_mean * chunks);
   // Items (surrogate rows head-major, then mean rows) from a counter, so that CTAs started
   // early (on SMs freed early) do more of them.
   for (;;) {

@@ -120,7 +120,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) cheap_heads_tc_kernel(const __g
   const int T = (a.N + kTcTile - 1) / kTcTile;
   const int surr_items = n_surr * T;
   const int Tm = (a.N + kMeanRows - 1) / kMeanRows;  // mean items per head
-  const int items = surr_items + n_mean * Tm;
+  // Mean heads folded into W_O's bias (skip_mean_y) need no rows of Y.
+  const int items = surr_items + (a.skip_mean_y ? 0 : n_mean * Tm);
 
   if (tid == 0) {
     for (int s = 0; s < kTcStages; ++s) {

@@ -39,6 +39,7 @@ struct RouterScratch {
   float* fa_part;               // [kFaTailUnits][4 chains][128 rows][64] split-tail partial O
   float* fa_stats;              // [kFaTailUnits][4 chains][128 rows][4] (m, l, xmax, -)
   unsigned int* fa_count;       // [kFaTailUnits][4 chains][4 quarters] split arrivals
+  float* wo_bias;               // [kMaxHeads * 64] W_O bias with the mean heads folded in
 };
 
 // Full attention splits the work items of its last, partial round along the keys over the
@@ -127,6 +128,7 @@ struct HeadAttnArgs {
   unsigned int* fa_count;       // zeroed by the launcher
   unsigned int* err;
   unsigned int* cheap_counter;  // one word of scratch, zeroed by the launcher
+  int skip_mean_y;              // 1: the mean heads' rows of Y are not written (folded into W_O)
 };
 
 // Full-mode heads (attn_full.cu).
@@ -175,8 +177,21 @@ struct LinearArgs {
   const float2* rope_cs;  // NULL: no RoPE
   int tok_per_view, patch_start, grid_w;
   const int32_t* tok_index;  // RoPE: token index of output row r (merged tokens), or NULL (r)
+  // K-blocks left out (W_O with mean heads folded into its bias): the 64-column blocks kb =
+  // skip_ids[skip_off[0] .. skip_off[1]) of A and W contribute nothing (K == 64 x blocks <=
+  // 32 x 64; no LayerNorm fold, no qk columns).  NULL: none.
+  const int32_t* skip_ids;
+  const int32_t* skip_off;
 };
 cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st);
+
+// W_O's bias with the mean heads folded in (Algorithm 1, step 3): a mean head's output is the
+// same row mu_h = bf16(mean_v[h]) for every token, so its part of Y W_O^T is one vector:
+//   bias_out[n] = b_o[n] + sum over mean heads h of sum_k mu_h[k] W_O[n][64 h + k]
+// (mean heads: head_ids[offsets[0] .. offsets[1]); b_o NULL: 0).  W_O [D][H 64] bf16.
+cudaError_t launch_wo_mean_fold(int D, int H, const __nv_bfloat16* w_o, const float* b_o,
+                                const float* mean_v, const int32_t* head_ids,
+                                const int32_t* offsets, float* bias_out, cudaStream_t st);
 
 // Per-row LayerNorm statistics as (mean, M2) of 128-column blocks: x [M][D] bf16 ->
 // part [M][D / 128] float2 (D % 256 == 0, D <= 4096).

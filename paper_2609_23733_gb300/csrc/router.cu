@@ -612,7 +612,7 @@ cudaError_t launch_wait_selftest(unsigned int* err, unsigned long long limit_ns,
 
 size_t heads_scratch_bytes(int H) {
   return router_scratch_bytes(H) + (size_t)kMaxHeads * kLinState * 4 +
-         (kFaPartFloats + kFaStatsFloats + kFaCountWords) * 4;
+         (kFaPartFloats + kFaStatsFloats + kFaCountWords) * 4 + (size_t)kMaxHeads * 64 * 4;
 }
 
 RouterScratch carve_router_scratch(void* ws, int H) {
@@ -646,6 +646,7 @@ RouterScratch carve_router_scratch(void* ws, int H) {
   sc.fa_part = sc.lin_state + (size_t)kMaxHeads * kLinState;
   sc.fa_stats = sc.fa_part + kFaPartFloats;
   sc.fa_count = reinterpret_cast<unsigned int*>(sc.fa_stats + kFaStatsFloats);
+  sc.wo_bias = reinterpret_cast<float*>(sc.fa_count + kFaCountWords);
   return sc;
 }
 
