@@ -63,6 +63,9 @@ struct GemmParams {
   const int32_t* skip_off;
 };
 
+// kSkip: the instance that leaves K-blocks out (GemmParams::skip_ids); the other instance has
+// none of that bookkeeping.
+template <bool kSkip>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a,
                 const __grid_constant__ CUtensorMap tmap_b,
@@ -90,7 +93,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&sm.drain, 1);
     sm.abort_flag = 0;
     uint32_t skip = 0;
-    if (prm.skip_ids) {
+    if (kSkip) {
       const int s0 = __ldg(prm.skip_off), s1 = __ldg(prm.skip_off + 1);
       for (int i = s0; i < s1; ++i) skip |= 1u << (__ldg(prm.skip_ids + i) & 31);
     }
@@ -109,9 +112,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = __shfl_sync(0xffffffffu, sm.tmem_base, 0);
-  // K-blocks left out, and whether that is all of them (the accumulator is then 0).
-  const uint32_t skip = sm.skip_mask;
-  const bool acc_zero = skip != 0 && __popc(skip & (k_blocks >= 32 ? 0xffffffffu : (1u << k_blocks) - 1u)) == k_blocks;
+  // K-blocks left out, and whether that is all of them (A W^T is then 0).
+  const uint32_t skip = kSkip ? sm.skip_mask : 0u;
+  const bool acc_zero = kSkip && skip != 0 && __popc(skip & (k_blocks >= 32 ? 0xffffffffu : (1u << k_blocks) - 1u)) == k_blocks;
 
   if (warp == 0) {
     // TMA producer: converged warp (warp-uniform coordinates), one elected lane issues.
@@ -120,7 +123,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
       const int mt = t / n_tiles, nt = t - mt * n_tiles;
       for (int kb = 0; kb < k_blocks; ++kb) {
-        if ((skip >> kb) & 1u) continue;
+        if (kSkip && ((skip >> kb) & 1u)) continue;
         const int st = lc % kStages;
         ok = mbar_wait_warp(&sm.empty[st], ((lc / kStages) & 1) ^ 1, prm.err, abort_flag);
         if (!ok) break;
@@ -155,7 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t d = tmem + ab * kBN;
       bool first = true;  // the tile's first MMA overwrites the accumulator
       for (int kb = 0; kb < k_blocks; ++kb) {
-        if ((skip >> kb) & 1u) continue;
+        if (kSkip && ((skip >> kb) & 1u)) continue;
         const int st = lc % kStages;
         ok = mbar_wait_warp(&sm.full[st], (lc / kStages) & 1, prm.err, abort_flag);
         if (!ok) break;
@@ -165,7 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
-            tc_mma_ss(d, da + 2 * kk, db + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
+            tc_mma_ss(d, da + 2 * kk, db + 2 * kk, idesc, ((kSkip ? !first : kb > 0) || kk > 0) ? 1u : 0u);
           tc_commit(&sm.empty[st]);
         }
         __syncwarp();
@@ -189,6 +192,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int half = e >> 2;                // column half of the tile
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
     unsigned char* stg = reinterpret_cast<unsigned char*>(&sm.stage[e][0][0]);
+    if (acc_zero) {
+      // Every K-block is left out, so no MMA writes the accumulators: zero this thread's
+      // columns of both once, and every tile then reads A W^T = 0.
+      float z[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k) z[k] = 0.f;
+#pragma unroll
+      for (int ab = 0; ab < 2; ++ab)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tmem_st32(t_lane + ab * kBN + half * 128 + 32 * q, z);
+      tmem_wait_st();
+    }
     uint32_t i = 0, nst = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++i) {
       const int mt = t / n_tiles, nt = t - mt * n_tiles;
@@ -396,10 +411,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int cc = 0; cc < 4; ++cc) {
         if (cc + 1 < 4) tmem_ld32(tcol + 32 * (cc + 1), v[(cc + 1) & 1]);  // in flight meanwhile
         float* x = v[cc & 1];
-        if (acc_zero) {  // every K-block left out: A W^T is 0 (TMEM was not written)
-#pragma unroll
-          for (int k = 0; k < 32; ++k) x[k] = 0.f;
-        }
         const int col0 = nt * kBN + half * 128 + cc * 32;
         if (col0 < N) {
           // Bias, GELU, LayerScale and residual on column pairs (packed f32x2 arithmetic).
@@ -548,7 +559,9 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
   e = make_tmap_bf16_2d(&to, a.out, (uint64_t)a.N, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 64);
   if (e != cudaSuccess) return e;
   const int smem = (int)sizeof(GemmSmem) + 1024;
-  e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  const bool skip = a.skip_ids != nullptr;
+  e = cudaFuncSetAttribute(skip ? gemm_kernel<true> : gemm_kernel<false>,
+                           cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int tiles = ((a.M + kBM - 1) / kBM) * ((a.N + kBN - 1) / kBN);
   if ((a.ln_part && (a.K % 256 != 0 || !a.ln_c || !a.bias)) ||
@@ -566,7 +579,10 @@ cudaError_t launch_linear(const LinearArgs& a, int num_sms, cudaStream_t st) {
                  qk ? a.qk_cols : 0, a.qn_g, a.qn_b, a.kn_g, a.kn_b, a.qk_eps, a.rope_cs,
                  a.tok_per_view, a.patch_start, a.grid_w, a.tok_index, a.skip_ids, a.skip_off};
   prof_before(VP_KERNEL_GEMM, st);
-  gemm_kernel<<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
+  if (skip)
+    gemm_kernel<true><<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
+  else
+    gemm_kernel<false><<<min(num_sms, tiles), kThreads, smem, st>>>(ta, tb, to, prm);
   prof_after(st);
   return cudaGetLastError();
 }
