@@ -11,6 +11,9 @@
 // bias / GELU / LayerScale / residual, packs bf16 into a 64-byte-swizzled 32 x 32 staging
 // block in shared memory and writes it with a TMA tensor store (clipped at the tensor edge).
 // Tiles are visited N-fastest so the CTAs in flight share A rows and all of W in L2.
+// A second instance (kSkip) leaves chosen 64-column K-blocks out: W_O with the mean heads
+// folded into its bias (wo_mean_fold_kernel) skips their copies and MMAs, and with every block
+// left out it is its epilogue alone.
 #include <math.h>
 
 #include "common.cuh"
