@@ -1,6 +1,6 @@
 """Host logic of bench.py's router-vs-exact saliency report (CPU): the rank correlation
 against scipy's Spearman, the routing of a saliency against the oracle's §4.2 rule, and the
-route table's bookkeeping."""
+route table's bookkeeping, and the roofline's fraction of the burst peak."""
 import numpy as np
 import pytest
 from scipy.stats import spearmanr
@@ -35,3 +35,13 @@ def test_saliency_agreement_table():
     assert rep["route_table"] == [[2, 0, 0], [1, 0, 0], [0, 1, 1]]
     assert rep["routes_agree"] == 3
     assert np.isclose(rep["spearman"], spearmanr(s_router, s_exact).statistic)
+
+
+def test_burst_fraction_of_the_roofline():
+    pk = {"bf16_tflops": 2000.0, "bf16_tflops_sustained": 1600.0,
+          "clocks_under_load": {"sm_mhz_median": 1500.0}}
+    out = bench.burst_fraction(pk, 1200.0)
+    assert out == {"peak_burst": 2000.0, "frac_of_burst": 0.6, "peak_sustained_sm_mhz": 1500.0}
+    assert bench.burst_fraction({}, 1200.0) == {}
+    assert bench.burst_fraction({"bf16_tflops": 1000.0}, 500.0) == {"peak_burst": 1000.0,
+                                                                      "frac_of_burst": 0.5}
